@@ -1,0 +1,66 @@
+"""Plant plausible mistakes in copies of the oracle and check that the pins catch each one.
+
+Every mutant is a one-token edit of ``oracle/wino_oracle.c`` (a dropped term,
+a flipped sign or comparison, a wrong index, a transposed row kind, a lost
+rule), compiled on the CPU into a temporary library and run through the
+pins of ``oracle_pins``; at least one pin must fail for every mutant.
+"""
+import shutil
+import subprocess
+from pathlib import Path
+
+import pytest
+
+import oracle
+from oracle_pins import ALL_PINS
+
+SRC = Path(oracle.__file__).resolve().parent / "wino_oracle.c"
+
+# (name, text in the oracle, replacement)
+MUTANTS = [
+    ("draft_not_strict", "(pmax[row_blk + l] > tau1)", "(pmax[row_blk + l] >= tau1)"),
+    ("verify_not_strict", "(ptarget[row_shd + l] < tau2)", "(ptarget[row_shd + l] <= tau2)"),
+    ("draft_reads_shadow_row", "(pmax[row_blk + l] > tau1)", "(pmax[row_shd + l] > tau1)"),
+    ("verify_reads_block_row", "(ptarget[row_shd + l] < tau2)", "(ptarget[row_blk + l] < tau2)"),
+    ("draft_ignores_mask_state", "inD[l] = (prev[l] == mask_id) && ", "inD[l] = "),
+    ("verify_ignores_mask_state", "inR[l] = (prev[l] != mask_id) && ", "inR[l] = "),
+    ("no_fallback", "if (n_draft == 0 && n_mask > 0) {", "if (0) {"),
+    ("fallback_last_on_ties", "pmax[row_blk + l] > best)) {", "pmax[row_blk + l] >= best)) {"),
+    ("fallback_ignores_mask_state", "if (prev[l] == mask_id && (fallback < 0", "if ((fallback < 0"),
+    ("argmax_last_on_ties", "if (logit[v] > m) {", "if (logit[v] >= m) {"),
+    ("softmax_drops_term", "for (int64_t v = 0; v < V; ++v)\n                Z += exp",
+     "for (int64_t v = 1; v < V; ++v)\n                Z += exp"),
+    ("softmax_sign_flip", "Z += exp(logit[v] - m);", "Z += exp(m - logit[v]);"),
+    ("pmax_not_inverted", "pmax[n] = 1.0 / Z;", "pmax[n] = Z / V;"),
+    ("ptarget_uses_argmax", "exp(logit[t] - m) / Z", "exp(logit[a] - m) / Z"),
+    ("hidden_index_reversed", "oracle_bf16_to_double(h[k]) *", "oracle_bf16_to_double(h[d - 1 - k]) *"),
+    ("bf16_wrong_shift", "(uint32_t)bits << 16;", "(uint32_t)bits << 15;"),
+    ("verify_target_on_block_row", "target[(s * 2 + 1) * blk_len + l] = (y == mask_id) ? -1 : y;",
+     "target[(s * 2 + 0) * blk_len + l] = (y == mask_id) ? -1 : y;"),
+    ("remask_not_counted", "++remasked;", ""),
+    ("left_counts_old_state", "left += (y[l] == mask_id);", "left += (prev[l] == mask_id);"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_kill_mutant(tmp_path, name, old, new):
+    src = SRC.read_text()
+    assert src.count(old) >= 1, f"mutation site for {name} not found"
+    mutated = src.replace(old, new, 1)
+    c = tmp_path / "mutant.c"
+    c.write_text(mutated)
+    so = tmp_path / f"liboracle_{name}.so"
+    gcc = shutil.which("gcc")
+    assert gcc
+    r = subprocess.run([gcc, "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared", "-fopenmp", str(c),
+                        "-o", str(so), "-lm"], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    O = oracle.Oracle(str(so))
+    failed = []
+    for pin in ALL_PINS:
+        try:
+            pin(O)
+        except AssertionError:
+            failed.append(pin.__name__)
+            break
+    assert failed, f"no pin caught mutant {name}"
