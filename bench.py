@@ -1,0 +1,380 @@
+#!/usr/bin/env python3
+"""Throughput of one WINO step (fused LM head + vocabulary softmax + Eq. 4 revoke) on GB300.
+
+Workload: the LLaDA-8B-shaped single step (d=4096, V=126464, one sequence,
+block of 128 plus 128 shadow rows: N=256 scored rows), seeded synthetic
+inputs (wino_synth).  A step is one wino_step call through the C ABI: the
+fused score kernel, the cross-tile merge and the draft/verify kernel.
+
+Prints one JSON line (rank 0).  `value` is scored rows/s over the K timed
+steps with inputs resident in HBM (W is 1.04 GB, larger than L2, so no L2
+flush is needed); `e2e` is the same metric with each step's hidden states
+and token state copied in from pinned host memory and the tokens and counts
+copied back, through the same C ABI; `roofline` rates the dominant kernel
+(the fused score kernel, timed by CUDA events the library records around
+each launch on the launch stream) against the measured HBM copy bandwidth;
+`cpu_baseline` times the fp64 CPU oracle on a bounded sample of the same
+workload on this host's cores.
+
+--impl reference times the oracle itself as the reference arm (CPU, fp64).
+Multi-GPU (torchrun): every rank decodes its own replica (weak scaling); no
+collective on the data path.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "scored rows/s for fused LM-head+softmax+WINO revoke; % of GEMM/HBM roofline"
+UNIT = "rows/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured (MEASURED_PEAKS.json)"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def config_dict(w):
+    return {"workload": w.name, "N": w.N, "d": w.d, "V": w.V, "n_seq": w.n_seq, "blk_len": w.blk_len,
+            "tau1": w.tau1, "tau2": w.tau2, "seed": w.seed,
+            "l2": "inputs larger than L2: W_lm is %.3f GB, read once per step" % (w.V * w.d * 2 / 1e9),
+            "parallelism": "replicas (one independent decode per GPU)"}
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock, power and throttle reasons while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str | None):
+        self.samples = []
+        self.proc = None
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50"]
+        if gpu_id:
+            cmd += ["-i", gpu_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        if not self.samples:
+            return None
+        inside = [s for t, s in self.samples if t0 <= t <= t1 + 0.06]
+        used = inside or [min(self.samples, key=lambda ts: min(abs(ts[0] - t0), abs(ts[0] - t1)))[1]]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, pw, reasons = [], [], [], set()
+        for s in used:
+            try:
+                sm.append(float(s[0]))
+                mx.append(float(s[1]))
+                pw.append(float(s[2]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, s[3:]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "power_w_max": max(pw), "reasons": sorted(reasons),
+                "samples": len(sm), "samples_in_timed_region": len(inside)}
+
+
+def gpu_uuid(dev):
+    import torch
+    try:
+        u = torch.cuda.get_device_properties(dev).uuid
+        s = str(u)
+        return s if s.startswith("GPU-") else "GPU-" + s
+    except Exception:
+        return None
+
+
+def oracle_cpu_baseline(w, W, H, targets, budget_s: float = 12.0, max_rows: int = 256):
+    """Time the oracle scoring rows of this step in batches of one row per thread until the budget is spent."""
+    import numpy as np
+
+    import oracle
+    nt = oracle.num_threads()
+    rows, t_total, i = 0, 0.0, 0
+    while rows < max_rows and (t_total < budget_s or rows == 0):
+        idx = np.arange(i, i + nt) % w.N
+        t0 = time.perf_counter()
+        oracle.score_rows(H[idx], W, targets[idx])
+        t_total += time.perf_counter() - t0
+        rows += nt
+        i += nt
+    return {"value": rows / t_total, "unit": UNIT, "cores": nt, "kind": "oracle",
+            "sample": f"{rows} of the {w.N} rows of one step of {w.name}, each scored over the full vocabulary "
+                      f"in fp64 ({t_total:.1f} s); the Eq. 4 update (microseconds) is not included",
+            "seconds": t_total}
+
+
+def run_reference(args):
+    """Reference arm: the fp64 oracle as it stands, on this host's cores, same workload and metric."""
+    import numpy as np
+
+    import oracle
+    import wino_synth as ws
+    w = ws.WORKLOADS[args.workload]
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    H = ws.hidden_states(w, W, st, step=0)
+    t = oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
+    nt = oracle.num_threads()
+    # calibrate: one batch of nt rows over a vocabulary slice
+    slice_v = min(w.V, 4096)
+    t0 = time.perf_counter()
+    oracle.score_rows(H[:nt], W[:slice_v], t[:nt])
+    per_logit = (time.perf_counter() - t0) / (nt * slice_v)
+    per_step = max(0.005, args.ref_budget_s / (args.steps + args.warmup))
+    # rows x vocabulary-slice sample per step sized to the per-step budget (at least one row-slice per thread)
+    sv = int(min(w.V, max(256, per_step / (per_logit * nt))))
+    sample_logits = nt * sv
+    times = []
+    for i in range(args.warmup + args.steps):
+        idx = (np.arange(nt) + i * nt) % w.N
+        v0 = (i * 7919) % max(1, w.V - sv + 1)
+        t0 = time.perf_counter()
+        oracle.score_rows(H[idx], W[v0:v0 + sv], None)
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append(dt)
+    tot = sum(times)
+    rows_equiv = args.steps * sample_logits / w.V
+    value = rows_equiv / tot
+    sample = (f"per step {nt} rows x a {sv}-entry vocabulary slice ({sample_logits / w.V:.4f} full-vocabulary rows) "
+              f"of {w.name}, fp64 oracle; value counts full-vocabulary-row equivalents")
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(w), "impl": "reference",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": nt, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+
+
+def run_wino(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+
+    from paper_2605_16941_gb300 import build as pkg_build
+    if rank == 0:
+        pkg_build.build()
+    if world > 1:
+        dist.barrier()
+    import paper_2605_16941_gb300 as wino
+    import wino_synth as ws
+
+    w = ws.WORKLOADS[args.workload]
+    t_gen = time.time()
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    n_h = 4
+    Hs = [ws.hidden_states(w, W, st, step=k) for k in range(n_h)]
+    log(f"[rank {rank}] inputs generated in {time.time() - t_gen:.1f} s")
+
+    def to_dev(a):
+        a = np.ascontiguousarray(a)
+        return torch.from_numpy(a.view(np.int16) if a.dtype == np.uint16 else a).to(dev)
+
+    Wd = to_dev(W)
+    Hd = [to_dev(h) for h in Hs]
+    tok = to_dev(st.tokens)
+    counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device=dev)
+    wsp = wino.workspace(w.N, w.d, w.V, device=dev)
+    p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len)
+    stream = torch.cuda.current_stream(dev)
+    sid = stream.cuda_stream
+
+    def step(i):
+        wino.wino_step(Hd[i % n_h], Wd, tok, p, counts, wsp, stream=sid)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize(dev)
+    if wino.wino_read_device_status(wsp, stream=sid) != wino.WINO_OK:
+        raise RuntimeError("device status not OK after warm-up")
+
+    clocks = ClockSampler(gpu_uuid(dev)) if rank == 0 else None
+    time.sleep(0.3 if clocks else 0)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    wino.wino_profile_begin(args.steps)
+    tw0 = time.time()
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    tw1 = time.time()
+    score_ms, score_n = wino.wino_profile_end()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    if clocks:
+        time.sleep(0.1)
+        clocks.stop()
+    if wino.wino_read_device_status(wsp, stream=sid) != wino.WINO_OK:
+        raise RuntimeError("device status not OK after the timed region")
+    t_max = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
+    t_max = float(t_max.item())
+
+    # ---- end to end through the C ABI with host buffers (pinned), one host read of the result per step
+    Hh = [torch.from_numpy(np.ascontiguousarray(h).view(np.int16)).pin_memory() for h in Hs]
+    tok_h = torch.from_numpy(st.tokens).pin_memory()
+    tok_out = torch.empty_like(tok_h).pin_memory()
+    cnt_out = torch.empty((w.n_seq, 3), dtype=torch.int32).pin_memory()
+    Hbuf = torch.empty_like(Hd[0])
+    e2e_steps = args.steps
+
+    def e2e_step(i):
+        Hbuf.copy_(Hh[i % n_h], non_blocking=True)
+        tok.copy_(tok_h, non_blocking=True)
+        wino.wino_step(Hbuf, Wd, tok, p, counts, wsp, stream=sid)
+        tok_out.copy_(tok, non_blocking=True)
+        cnt_out.copy_(counts, non_blocking=True)
+        stream.synchronize()
+
+    for i in range(max(3, args.warmup)):
+        e2e_step(i)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    te0 = time.perf_counter()
+    for i in range(e2e_steps):
+        e2e_step(i)
+    torch.cuda.synchronize(dev)
+    te = time.perf_counter() - te0
+    te_t = torch.tensor([te], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(te_t, op=dist.ReduceOp.MAX)
+    te = float(te_t.item())
+    h2d = Hh[0].numel() * 2 + tok_h.numel() * 4
+    d2h = tok_out.numel() * 4 + cnt_out.numel() * 4
+
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+
+    peaks, peak_src = load_peaks()
+    flops = 2.0 * w.N * w.d * w.V
+    w_bytes = w.V * w.d * 2.0
+    h_bytes = w.N * w.d * 2.0
+    alg_bytes = w_bytes + h_bytes + 12.0 * w.N
+    t_flop = flops / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = alg_bytes / (peaks["hbm_gbs"] * 1e9)
+    bound = "hbm" if t_hbm >= t_flop else "tensor"
+    score_avg_s = (score_ms / max(1, score_n)) / 1e3
+    if bound == "hbm":
+        achieved, peak, unit = alg_bytes / score_avg_s / 1e9, peaks["hbm_gbs"], "GB/s"
+    else:
+        achieved, peak, unit = flops / score_avg_s / 1e12, peaks["bf16_tflops"], "TFLOP/s"
+    step_s = t_max / 1e3 / args.steps
+    value = world * w.N * args.steps / (t_max / 1e3)
+    clock_info = clocks.summary(tw0, tw1) if clocks else None
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        import oracle
+        t = oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
+        cpu = oracle_cpu_baseline(w, W, Hs[0], t, budget_s=args.cpu_budget_s)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_dict(w),
+        "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                     "traffic": None, "kernel": "score_kernel (fused LM-head GEMM + online vocab softmax)",
+                     "algorithmic_per_launch": {"bytes": alg_bytes, "flops": flops},
+                     "avg_launch_us": score_avg_s * 1e6, "launches_timed": score_n, "peak_source": peak_src,
+                     "tensor_tflops": flops / score_avg_s / 1e12,
+                     "tensor_frac": flops / score_avg_s / 1e12 / peaks["bf16_tflops"]},
+        "step_roofline_frac": max(t_flop, w_bytes / (peaks["hbm_gbs"] * 1e9)) / step_s,
+        "tflops_per_step": flops / step_s / 1e12,
+        "e2e": {"value": world * w.N * e2e_steps / te, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * te / e2e_steps},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clock_info,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["wino", "reference"], default="wino")
+    ap.add_argument("--workload", default="llada_b1")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget-s", type=float, default=12.0)
+    ap.add_argument("--ref-budget-s", type=float, default=90.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args)
+        return
+    run_wino(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

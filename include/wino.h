@@ -1,0 +1,157 @@
+/*
+ * wino.h -- C ABI of the GB300 (sm_103a) WINO scoring-and-revoke step.
+ *
+ * WINO ("Wide-In, Narrow-Out", arXiv 2605.16941, Sec. 4) decodes a block of a
+ * diffusion LLM's response by drafting and verifying in one forward pass.
+ * Per step and per sequence it scores 2*L_b rows of hidden states through
+ * the LM head: L_b rows of the current block Y_cur (drafting, Eq. 2) and L_b
+ * rows of the shadow block Y_shad (verification, Eq. 3), then applies Eq. 4:
+ *   - a masked position whose block row has max_v p > tau1 takes that row's
+ *     argmax token (Eq. 2); if no masked position clears tau1, the single
+ *     most confident masked position is drafted anyway (greedy rule, Eq. 1);
+ *   - a decoded position whose shadow row gives its current token a
+ *     probability < tau2 is re-masked (Eq. 3);
+ *   - everything else, and every position outside the block, is unchanged.
+ *
+ * Conventions shared by every entry point
+ *   - Every array argument is a DEVICE pointer owned by the caller; the
+ *     library never allocates, frees or synchronises (except
+ *     wino_read_device_status, which reads back one word).
+ *   - bf16 data are passed as uint16_t bit patterns (IEEE binary32 top half).
+ *   - Row order of the scored rows is [s][kind][l]: sequence s, kind 0 = the
+ *     current-block row of position l, kind 1 = its shadow-block row; row
+ *     index n = (2*s + kind)*blk_len + l, N = 2*n_seq*blk_len.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream); all work is
+ *     enqueued on it asynchronously, in order.
+ *   - Return value: WINO_OK (0) or a negative wino_status.  On an argument
+ *     error nothing is enqueued.  Device-side failures (a bounded wait that
+ *     expired) are reported in the workspace status word, see
+ *     wino_read_device_status.
+ *   - Devices: compute capability 10.3 (GB300).  Other devices get
+ *     WINO_ERR_UNSUPPORTED.
+ */
+#ifndef WINO_H
+#define WINO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define WINO_API __attribute__((visibility("default")))
+#else
+#define WINO_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    WINO_OK = 0,
+    WINO_ERR_ARG = -1,            /* null pointer, misaligned pointer, threshold out of range  */
+    WINO_ERR_SHAPE = -2,          /* sizes outside the supported range (see each call)         */
+    WINO_ERR_WORKSPACE = -3,      /* ws_bytes below wino_workspace_size()                      */
+    WINO_ERR_CUDA = -4,           /* a CUDA runtime/driver call or kernel launch failed        */
+    WINO_ERR_MAX_STEPS = -5,      /* a decode loop exceeded its step budget (loop drivers)     */
+    WINO_ERR_DEVICE_TIMEOUT = -6, /* a bounded device-side wait expired; outputs are invalid   */
+    WINO_ERR_UNSUPPORTED = -7     /* not a compute-capability 10.3 device                      */
+} wino_status;
+
+/* Decoding parameters (host memory, read during the call only). */
+typedef struct {
+    float tau1;        /* drafting threshold, Eq. 2: draft iff max_v p > tau1 (strict)          */
+    float tau2;        /* verification threshold, Eq. 3: re-mask iff p(current) < tau2 (strict) */
+    int32_t mask_id;   /* the [MASK] token id, in [0, V)                                         */
+    int32_t n_seq;     /* sequences in the batch                                                 */
+    int32_t seq_len;   /* S: length of each row of `tokens`                                      */
+    int32_t blk_start; /* first position of the current block Y_cur                             */
+    int32_t blk_len;   /* L_b, 1..1024; blk_start + blk_len <= seq_len                           */
+    int32_t max_steps; /* step budget for loop drivers; unused by the calls below               */
+} wino_params;
+
+/*
+ * Bytes of scratch the score path needs for N rows of dimension d over a
+ * vocabulary of V entries (per-tile partial softmax statistics, targets and
+ * per-row results, plus one status word).  `ws` passed to wino_score_rows /
+ * wino_step must hold at least this many bytes and be 256-byte aligned.
+ * Returns WINO_ERR_SHAPE for sizes the kernels do not support, see
+ * wino_score_rows.
+ */
+WINO_API int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes);
+
+/*
+ * Fused LM-head GEMM + full-vocabulary softmax statistics (the p_theta(.|Y~)
+ * of Eq. 2 and Eq. 3), without writing the [N, V] logits anywhere.
+ *   H       [N, d] bf16, row-major, 16-byte aligned      (hidden states)
+ *   W       [V, d] bf16, row-major, 16-byte aligned      (LM-head weights)
+ *   target  [N] int32 or NULL: token whose probability is wanted per row;
+ *           a value outside [0, V) means "none"
+ *   argmax  [N] int32 out: argmax_v l_v, the smallest v among exact ties
+ *   pmax    [N] float out: max_v p_v = 1 / sum_v exp(l_v - max_u l_u)
+ *   ptarget [N] float out: p_target, 0 where the row has no target
+ * Shapes: 1 <= N <= 2^24, 8 <= d <= 65536 with d % 8 == 0, 2 <= V <= 2^27.
+ * Logits are accumulated in fp32 on the tensor cores; the softmax runs in
+ * fp32.  The status word in `ws` is cleared at the start of the call.
+ */
+WINO_API int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V,
+                    const int32_t *target, int32_t *argmax, float *pmax, float *ptarget, void *ws,
+                    size_t ws_bytes, void *stream);
+
+/*
+ * Eq. 4 on every sequence's current block, in place on tokens[n_seq, seq_len]
+ * (int32), from per-row statistics in [s][kind][l] order (argmax/pmax of the
+ * kind-0 rows drive drafting; ptarget of the kind-1 rows, i.e. the
+ * probability of the position's CURRENT token, drives verification).
+ *   counts [n_seq, 3] int32 out: {drafted (MASK -> token), re-masked,
+ *                                MASKs left in the block after the step}
+ *   flags  [n_seq, blk_len] int8 out or NULL: per position 0 unchanged,
+ *          1 drafted (pmax > tau1), 2 drafted by the at-least-one rule,
+ *          3 re-masked, 4 selected for drafting but its argmax is MASK itself
+ *          (the position stays MASK and is not counted as drafted)
+ * Ties in the at-least-one rule go to the smallest position.  Requires
+ * 0 <= tau1, tau2 <= 1, 1 <= blk_len <= 1024, n_seq >= 1.
+ */
+WINO_API int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
+                      const wino_params *p, int32_t *counts, int8_t *flags, void *stream);
+
+/*
+ * One whole WINO step: targets of the shadow rows are gathered from `tokens`
+ * (the current token of each decoded position, none for masked positions and
+ * for block rows), every row is scored as in wino_score_rows, and Eq. 4 is
+ * applied as in wino_draft_verify.
+ *   H [2*n_seq*blk_len, d] bf16 rows in [s][kind][l] order; W [V, d] bf16.
+ * If a device wait expired, tokens are left unchanged and every counts entry
+ * is set to WINO_ERR_DEVICE_TIMEOUT.
+ */
+WINO_API int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
+              int32_t *counts, int8_t *flags, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * Waits for `stream`, then reads the workspace status word written by the
+ * last score launch that used `ws`: WINO_OK, or WINO_ERR_DEVICE_TIMEOUT.
+ */
+WINO_API int wino_read_device_status(const void *ws, void *stream, int *device_status);
+
+/*
+ * Launch timing of the fused score kernel (for benchmarks).  Between
+ * wino_profile_begin(max_launches) and wino_profile_end, each of the first
+ * max_launches score launches (from wino_score_rows or wino_step) is
+ * bracketed by two CUDA events recorded on its stream; wino_profile_end
+ * waits for the last of them and returns the summed kernel time in
+ * milliseconds and the number of launches timed.  The events are created by
+ * begin and destroyed by end.  Only one profile may be open per process.
+ */
+WINO_API int wino_profile_begin(int max_launches);
+WINO_API int wino_profile_end(double *score_ms_total, int *score_launches);
+
+/* Static description of a status code. */
+WINO_API const char *wino_status_string(int status);
+
+/* Library version, (major << 16) | minor. */
+WINO_API int wino_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WINO_H */

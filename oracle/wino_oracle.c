@@ -48,16 +48,26 @@ double oracle_bf16_to_double(uint16_t bits)
     return (double)f;
 }
 
-/* Logits of one row: out[v] = sum_k h[k] * W[v, k], W row-major [V, d]. */
+/* Logits of one row: out[v] = sum_k h[k] * W[v, k], W row-major [V, d].
+ * The row h is widened to double once; the sum runs in index order. */
 void oracle_logits_row(const uint16_t *h, const uint16_t *W, int64_t d, int64_t V, double *out)
 {
+    double *hd = (double *)malloc((size_t)d * sizeof(double));
+    if (!hd) {
+        for (int64_t v = 0; v < V; ++v)
+            out[v] = NAN;
+        return;
+    }
+    for (int64_t k = 0; k < d; ++k)
+        hd[k] = oracle_bf16_to_double(h[k]);
     for (int64_t v = 0; v < V; ++v) {
         const uint16_t *w = W + v * d;
         double acc = 0.0;
         for (int64_t k = 0; k < d; ++k)
-            acc += oracle_bf16_to_double(h[k]) * oracle_bf16_to_double(w[k]);
+            acc += hd[k] * oracle_bf16_to_double(w[k]);
         out[v] = acc;
     }
+    free(hd);
 }
 
 /*

@@ -1,0 +1,168 @@
+"""ctypes binding of ``libwino.so`` (declared in ``include/wino.h``).
+
+Argument marshalling only: every function forwards to the C entry point of
+the same name, passing device pointers (``torch.Tensor.data_ptr()`` or raw
+integers), sizes and a ``cudaStream_t`` handle.  All computation happens in
+the library's CUDA kernels.  If the library has not been built, loading it
+raises ``RuntimeError``; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from pathlib import Path
+
+_LIB_PATH = Path(__file__).resolve().parent / "_build" / "libwino.so"
+_lib = None
+
+WINO_OK = 0
+WINO_ERR_ARG = -1
+WINO_ERR_SHAPE = -2
+WINO_ERR_WORKSPACE = -3
+WINO_ERR_CUDA = -4
+WINO_ERR_MAX_STEPS = -5
+WINO_ERR_DEVICE_TIMEOUT = -6
+WINO_ERR_UNSUPPORTED = -7
+
+# per-position outcome codes written to `flags`
+FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0, 1, 2, 3, 4
+
+EXPORTS = ("wino_workspace_size", "wino_score_rows", "wino_draft_verify", "wino_step",
+           "wino_read_device_status", "wino_profile_begin", "wino_profile_end", "wino_status_string",
+           "wino_version")
+
+
+class WinoError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {wino_status_string(status)} ({status})")
+
+
+class WinoParams(C.Structure):
+    _fields_ = [("tau1", C.c_float), ("tau2", C.c_float), ("mask_id", C.c_int32), ("n_seq", C.c_int32),
+                ("seq_len", C.c_int32), ("blk_start", C.c_int32), ("blk_len", C.c_int32),
+                ("max_steps", C.c_int32)]
+
+
+def library_path() -> Path:
+    return _LIB_PATH
+
+
+def lib() -> C.CDLL:
+    """Load libwino.so (built in-tree by ``__graft_entry__.build()``)."""
+    global _lib
+    if _lib is None:
+        if not _LIB_PATH.exists():
+            raise RuntimeError(f"{_LIB_PATH} is missing: build it with paper_2605_16941_gb300.build.build()")
+        L = C.CDLL(str(_LIB_PATH))
+        i64, vp, sz = C.c_int64, C.c_void_p, C.c_size_t
+        L.wino_workspace_size.restype = C.c_int
+        L.wino_workspace_size.argtypes = [i64, i64, i64, C.POINTER(sz)]
+        L.wino_score_rows.restype = C.c_int
+        L.wino_score_rows.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, vp, vp, sz, vp]
+        L.wino_draft_verify.restype = C.c_int
+        L.wino_draft_verify.argtypes = [vp, vp, vp, vp, C.POINTER(WinoParams), vp, vp, vp]
+        L.wino_step.restype = C.c_int
+        L.wino_step.argtypes = [vp, vp, i64, i64, vp, C.POINTER(WinoParams), vp, vp, vp, sz, vp]
+        L.wino_read_device_status.restype = C.c_int
+        L.wino_read_device_status.argtypes = [vp, vp, C.POINTER(C.c_int)]
+        L.wino_profile_begin.restype = C.c_int
+        L.wino_profile_begin.argtypes = [C.c_int]
+        L.wino_profile_end.restype = C.c_int
+        L.wino_profile_end.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_int)]
+        L.wino_status_string.restype = C.c_char_p
+        L.wino_status_string.argtypes = [C.c_int]
+        L.wino_version.restype = C.c_int
+        L.wino_version.argtypes = []
+        _lib = L
+    return _lib
+
+
+def _ptr(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(status: int, where: str) -> None:
+    if status != WINO_OK:
+        raise WinoError(status, where)
+
+
+def wino_status_string(status: int) -> str:
+    return lib().wino_status_string(int(status)).decode()
+
+
+def wino_version() -> int:
+    return lib().wino_version()
+
+
+def wino_workspace_size(N: int, d: int, V: int) -> int:
+    out = C.c_size_t(0)
+    _check(lib().wino_workspace_size(N, d, V, C.byref(out)), "wino_workspace_size")
+    return out.value
+
+
+def workspace(N: int, d: int, V: int, device=None):
+    """A zeroed uint8 device tensor of wino_workspace_size(N, d, V) bytes (allocated by PyTorch)."""
+    import torch
+    return torch.zeros(wino_workspace_size(N, d, V), dtype=torch.uint8, device=device or "cuda")
+
+
+def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
+                max_steps: int = 4096) -> WinoParams:
+    return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps)
+
+
+def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, N: int | None = None,
+                    d: int | None = None, V: int | None = None) -> None:
+    """Fused LM-head + full-vocabulary softmax statistics; shapes default to H.shape / W.shape."""
+    N = int(H.shape[0]) if N is None else N
+    d = int(H.shape[1]) if d is None else d
+    V = int(W.shape[0]) if V is None else V
+    ws_bytes = ws.numel() * ws.element_size()
+    _check(lib().wino_score_rows(_ptr(H), _ptr(W), N, d, V, _ptr(target), _ptr(argmax), _ptr(pmax), _ptr(ptarget),
+                                 _ptr(ws), ws_bytes, _stream(stream)), "wino_score_rows")
+
+
+def wino_draft_verify(tokens, argmax, pmax, ptarget, params: WinoParams, counts, flags=None, stream=None) -> None:
+    """Eq. 4 in place on ``tokens`` from per-row statistics."""
+    _check(lib().wino_draft_verify(_ptr(tokens), _ptr(argmax), _ptr(pmax), _ptr(ptarget), C.byref(params),
+                                   _ptr(counts), _ptr(flags), _stream(stream)), "wino_draft_verify")
+
+
+def wino_step(H, W, tokens, params: WinoParams, counts, ws, flags=None, stream=None, *, d: int | None = None,
+              V: int | None = None) -> None:
+    """One whole WINO step in place on ``tokens``."""
+    d = int(H.shape[1]) if d is None else d
+    V = int(W.shape[0]) if V is None else V
+    ws_bytes = ws.numel() * ws.element_size()
+    _check(lib().wino_step(_ptr(H), _ptr(W), d, V, _ptr(tokens), C.byref(params), _ptr(counts), _ptr(flags),
+                           _ptr(ws), ws_bytes, _stream(stream)), "wino_step")
+
+
+def wino_read_device_status(ws, stream=None) -> int:
+    out = C.c_int(0)
+    _check(lib().wino_read_device_status(_ptr(ws), _stream(stream), C.byref(out)), "wino_read_device_status")
+    return out.value
+
+
+def wino_profile_begin(max_launches: int) -> None:
+    _check(lib().wino_profile_begin(int(max_launches)), "wino_profile_begin")
+
+
+def wino_profile_end() -> tuple[float, int]:
+    """(summed score-kernel milliseconds, number of launches timed)."""
+    ms, n = C.c_double(0), C.c_int(0)
+    _check(lib().wino_profile_end(C.byref(ms), C.byref(n)), "wino_profile_end")
+    return ms.value, n.value

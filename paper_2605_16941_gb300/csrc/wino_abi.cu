@@ -1,0 +1,388 @@
+// wino_abi.cu -- the extern "C" entry points of libwino.so (see include/wino.h).
+//
+// Host side only: argument and shape checks, workspace layout, TMA tensor-map
+// encoding (cached), and kernel launches on the caller's stream.  No entry
+// point allocates device memory or synchronises, except
+// wino_read_device_status, which reads one status word back.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include <cudaTypedefs.h>  // PFN_cuTensorMapEncodeTiled
+
+#include "internal.h"
+
+namespace wino {
+namespace {
+
+constexpr int64_t kMaxN = int64_t(1) << 24;
+constexpr int64_t kMaxD = 65536;
+constexpr int64_t kMaxV = int64_t(1) << 27;
+constexpr size_t kAlign = 256;
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Workspace layout: [status | partial records [N][n_vt] | argmax[N] | pmax[N] | ptarget[N]].
+struct WsLayout {
+    size_t status, part, argmax, pmax, ptarget, total;
+};
+
+WsLayout ws_layout(int64_t N, int64_t V)
+{
+    const int64_t n_vt = (V + kBN - 1) / kBN;
+    WsLayout L{};
+    L.status = 0;
+    L.part = kAlign;
+    L.argmax = L.part + round_up((size_t)N * (size_t)n_vt * sizeof(float4), kAlign);
+    L.pmax = L.argmax + round_up((size_t)N * 4, kAlign);
+    L.ptarget = L.pmax + round_up((size_t)N * 4, kAlign);
+    L.total = L.ptarget + round_up((size_t)N * 4, kAlign);
+    return L;
+}
+
+bool shape_ok(int64_t N, int64_t d, int64_t V)
+{
+    return N >= 1 && N <= kMaxN && d >= 8 && d <= kMaxD && d % 8 == 0 && V >= 2 && V <= kMaxV;
+}
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ---------------------------------------------------------------- device facts
+
+struct DeviceInfo {
+    int sm_count = 0;
+    bool supported = false;
+};
+
+int device_info(DeviceInfo *out)
+{
+    static std::mutex mu;
+    static DeviceInfo cache[64];
+    static bool have[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+        return WINO_ERR_CUDA;
+    std::lock_guard<std::mutex> g(mu);
+    if (!have[dev]) {
+        int major = 0, minor = 0, sms = 0;
+        if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return WINO_ERR_CUDA;
+        cache[dev].sm_count = sms;
+        cache[dev].supported = (major == 10 && minor == 3);
+        have[dev] = true;
+    }
+    *out = cache[dev];
+    return out->supported ? WINO_OK : WINO_ERR_UNSUPPORTED;
+}
+
+// ---------------------------------------------------------------- tensor maps
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// A bf16 row-major [rows, cols] matrix read in boxes of box_rows x 64 with
+// 128-byte swizzling; out-of-range rows/columns read as zero.
+struct MapKey {
+    const void *ptr;
+    int64_t rows, cols;
+    int box_rows;
+    int dev;
+    bool operator==(const MapKey &o) const
+    {
+        return ptr == o.ptr && rows == o.rows && cols == o.cols && box_rows == o.box_rows && dev == o.dev;
+    }
+};
+
+int tensor_map(const void *ptr, int64_t rows, int64_t cols, int box_rows, CUtensorMap *out)
+{
+    static std::mutex mu;
+    constexpr int kSlots = 32;
+    static MapKey keys[kSlots];
+    static CUtensorMap maps[kSlots];
+    static int next = 0;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    const MapKey key{ptr, rows, cols, box_rows, dev};
+    std::lock_guard<std::mutex> g(mu);
+    for (int i = 0; i < kSlots; ++i)
+        if (keys[i] == key) {
+            *out = maps[i];
+            return WINO_OK;
+        }
+    auto fn = encode_fn();
+    if (!fn)
+        return WINO_ERR_CUDA;
+    CUtensorMap m;
+    std::memset(&m, 0, sizeof m);
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return WINO_ERR_CUDA;
+    keys[next] = key;
+    maps[next] = m;
+    next = (next + 1) % kSlots;
+    *out = m;
+    return WINO_OK;
+}
+
+// ---------------------------------------------------------------- launch timing
+
+// Optional timing of the score kernel: while enabled, every score launch is
+// bracketed by a pair of CUDA events recorded on the launch stream.
+struct Profiler {
+    std::mutex mu;
+    bool on = false;
+    int cap = 0, n = 0;
+    cudaEvent_t *ev = nullptr;
+} g_prof;
+
+void prof_record(int which, cudaStream_t stream)
+{
+    if (!g_prof.on)
+        return;
+    std::lock_guard<std::mutex> g(g_prof.mu);
+    if (!g_prof.on || g_prof.n >= g_prof.cap)
+        return;
+    cudaEventRecord(g_prof.ev[2 * g_prof.n + which], stream);
+    if (which == 1)
+        ++g_prof.n;
+}
+
+// ---------------------------------------------------------------- shared pieces
+
+int check_params(const wino_params *p)
+{
+    if (!p)
+        return WINO_ERR_ARG;
+    if (!(p->tau1 >= 0.f && p->tau1 <= 1.f) || !(p->tau2 >= 0.f && p->tau2 <= 1.f))
+        return WINO_ERR_ARG;
+    if (p->n_seq < 1 || p->blk_len < 1 || p->blk_len > kMaxBlkLen || p->blk_start < 0 || p->seq_len < 1 ||
+        (int64_t)p->blk_start + p->blk_len > p->seq_len || p->mask_id < 0)
+        return WINO_ERR_SHAPE;
+    if ((int64_t)p->n_seq * 2 * p->blk_len > kMaxN || (int64_t)p->n_seq * p->seq_len > (int64_t(1) << 31))
+        return WINO_ERR_SHAPE;
+    return WINO_OK;
+}
+
+// Score N rows into (argmax, pmax, ptarget); steps 1-2 of the WINO step.
+int score_into(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
+               int32_t *argmax, float *pmax, float *ptarget, void *ws, size_t ws_bytes, cudaStream_t stream)
+{
+    DeviceInfo info;
+    int rc = device_info(&info);
+    if (rc != WINO_OK)
+        return rc;
+    const WsLayout L = ws_layout(N, V);
+    if (ws_bytes < L.total)
+        return WINO_ERR_WORKSPACE;
+    CUtensorMap tmH, tmW;
+    if ((rc = tensor_map(H, N, d, kBM, &tmH)) != WINO_OK)
+        return rc;
+    if ((rc = tensor_map(W, V, d, kBN, &tmW)) != WINO_OK)
+        return rc;
+    uint8_t *w8 = static_cast<uint8_t *>(ws);
+    ScoreArgs a{};
+    a.N = (int32_t)N;
+    a.d = (int32_t)d;
+    a.V = (int32_t)V;
+    a.n_mb = (int32_t)((N + kBM - 1) / kBM);
+    a.n_vt = (int32_t)((V + kBN - 1) / kBN);
+    a.n_kb = (int32_t)((d + kBK - 1) / kBK);
+    a.n_tiles = (int64_t)a.n_mb * a.n_vt;
+    a.ts = ts;
+    a.part = reinterpret_cast<float4 *>(w8 + L.part);
+    a.status = reinterpret_cast<int32_t *>(w8 + L.status);
+    const int grid = (int)std::min<int64_t>(a.n_tiles, info.sm_count);
+    prof_record(0, stream);
+    if (launch_score(tmH, tmW, a, grid, stream) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    prof_record(1, stream);
+    if (launch_merge(a.part, a.N, a.n_vt, a.V, ts, a.status, argmax, pmax, ptarget, stream) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    return WINO_OK;
+}
+
+}  // namespace
+}  // namespace wino
+
+using namespace wino;
+
+extern "C" {
+
+int wino_version(void) { return (0 << 16) | 1; }
+
+const char *wino_status_string(int status)
+{
+    switch (status) {
+    case WINO_OK: return "ok";
+    case WINO_ERR_ARG: return "invalid argument (null or misaligned pointer, threshold outside [0, 1])";
+    case WINO_ERR_SHAPE: return "unsupported shape";
+    case WINO_ERR_WORKSPACE: return "workspace too small";
+    case WINO_ERR_CUDA: return "CUDA call or kernel launch failed";
+    case WINO_ERR_MAX_STEPS: return "decode loop exceeded its step budget";
+    case WINO_ERR_DEVICE_TIMEOUT: return "a bounded device-side wait expired; outputs are invalid";
+    case WINO_ERR_UNSUPPORTED: return "device is not compute capability 10.3";
+    default: return "unknown status";
+    }
+}
+
+int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
+{
+    if (!bytes)
+        return WINO_ERR_ARG;
+    if (!shape_ok(N, d, V))
+        return WINO_ERR_SHAPE;
+    *bytes = ws_layout(N, V).total;
+    return WINO_OK;
+}
+
+int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const int32_t *target,
+                    int32_t *argmax, float *pmax, float *ptarget, void *ws, size_t ws_bytes, void *stream)
+{
+    if (!H || !W || !argmax || !pmax || !ptarget || !ws)
+        return WINO_ERR_ARG;
+    if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign))
+        return WINO_ERR_ARG;
+    if (!shape_ok(N, d, V))
+        return WINO_ERR_SHAPE;
+    TargetSource ts{};
+    ts.target = target;
+    return score_into(H, W, N, d, V, ts, argmax, pmax, ptarget, ws, ws_bytes, static_cast<cudaStream_t>(stream));
+}
+
+int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
+                      const wino_params *p, int32_t *counts, int8_t *flags, void *stream)
+{
+    if (!tokens || !argmax || !pmax || !ptarget || !counts)
+        return WINO_ERR_ARG;
+    int rc = check_params(p);
+    if (rc != WINO_OK)
+        return rc;
+    DeviceInfo info;
+    if ((rc = device_info(&info)) != WINO_OK)
+        return rc;
+    if (launch_draft_verify(tokens, argmax, pmax, ptarget, *p, counts, flags, nullptr,
+                            static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    return WINO_OK;
+}
+
+int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
+              int32_t *counts, int8_t *flags, void *ws, size_t ws_bytes, void *stream)
+{
+    if (!H || !W || !tokens || !counts || !ws)
+        return WINO_ERR_ARG;
+    if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign))
+        return WINO_ERR_ARG;
+    int rc = check_params(p);
+    if (rc != WINO_OK)
+        return rc;
+    const int64_t N = (int64_t)p->n_seq * 2 * p->blk_len;
+    if (!shape_ok(N, d, V) || p->mask_id >= V)
+        return WINO_ERR_SHAPE;
+    const WsLayout L = ws_layout(N, V);
+    if (ws_bytes < L.total)
+        return WINO_ERR_WORKSPACE;
+    uint8_t *w8 = static_cast<uint8_t *>(ws);
+    int32_t *am = reinterpret_cast<int32_t *>(w8 + L.argmax);
+    float *pm = reinterpret_cast<float *>(w8 + L.pmax);
+    float *pt = reinterpret_cast<float *>(w8 + L.ptarget);
+    TargetSource ts{};
+    ts.tokens = tokens;
+    ts.seq_len = p->seq_len;
+    ts.blk_start = p->blk_start;
+    ts.blk_len = p->blk_len;
+    ts.mask_id = p->mask_id;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((rc = score_into(H, W, N, d, V, ts, am, pm, pt, ws, ws_bytes, s)) != WINO_OK)
+        return rc;
+    if (launch_draft_verify(tokens, am, pm, pt, *p, counts, flags, reinterpret_cast<const int32_t *>(w8 + L.status),
+                            s) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    return WINO_OK;
+}
+
+int wino_profile_begin(int max_launches)
+{
+    if (max_launches < 1 || max_launches > (1 << 20))
+        return WINO_ERR_ARG;
+    std::lock_guard<std::mutex> g(g_prof.mu);
+    if (g_prof.on)
+        return WINO_ERR_ARG;
+    g_prof.ev = new cudaEvent_t[2 * (size_t)max_launches];
+    for (int i = 0; i < 2 * max_launches; ++i)
+        if (cudaEventCreate(&g_prof.ev[i]) != cudaSuccess) {
+            for (int j = 0; j < i; ++j)
+                cudaEventDestroy(g_prof.ev[j]);
+            delete[] g_prof.ev;
+            g_prof.ev = nullptr;
+            return WINO_ERR_CUDA;
+        }
+    g_prof.cap = max_launches;
+    g_prof.n = 0;
+    g_prof.on = true;
+    return WINO_OK;
+}
+
+int wino_profile_end(double *score_ms_total, int *score_launches)
+{
+    if (!score_ms_total || !score_launches)
+        return WINO_ERR_ARG;
+    std::lock_guard<std::mutex> g(g_prof.mu);
+    if (!g_prof.on)
+        return WINO_ERR_ARG;
+    int rc = WINO_OK;
+    double total = 0.0;
+    for (int i = 0; i < g_prof.n; ++i) {
+        float ms = 0.f;
+        if (cudaEventSynchronize(g_prof.ev[2 * i + 1]) != cudaSuccess ||
+            cudaEventElapsedTime(&ms, g_prof.ev[2 * i], g_prof.ev[2 * i + 1]) != cudaSuccess)
+            rc = WINO_ERR_CUDA;
+        total += ms;
+    }
+    for (int i = 0; i < 2 * g_prof.cap; ++i)
+        cudaEventDestroy(g_prof.ev[i]);
+    delete[] g_prof.ev;
+    g_prof.ev = nullptr;
+    *score_ms_total = total;
+    *score_launches = g_prof.n;
+    g_prof.on = false;
+    g_prof.cap = g_prof.n = 0;
+    return rc;
+}
+
+int wino_read_device_status(const void *ws, void *stream, int *device_status)
+{
+    if (!ws || !device_status)
+        return WINO_ERR_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    int32_t v = 0;
+    if (cudaMemcpy(&v, ws, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    *device_status = v;
+    return WINO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,81 @@
+"""Semi-autoregressive WINO decode loop over the C ABI (Sec. 3 and Sec. 4.2.3).
+
+Blocks are decoded left to right; inside a block ``wino_step`` is repeated
+until no position of the block is MASK in any sequence of the batch.  The
+only device-to-host traffic per step is the [n_seq, 3] counts array, read to
+decide whether the block is finished.  The hidden states of each step come
+from a caller-supplied function (the transformer forward with the
+shadow-block attention mask is outside this library).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Callable
+
+from ._abi import WINO_ERR_MAX_STEPS, WinoError, make_params, wino_step, wino_workspace_size
+
+
+@dataclass
+class BlockStats:
+    block: int
+    blk_start: int
+    steps: int = 0
+    drafted: int = 0
+    remasked: int = 0
+    fallback_steps: int = 0  # steps on which some sequence drafted by the at-least-one rule only
+
+
+@dataclass
+class LoopStats:
+    blocks: list = field(default_factory=list)
+    total_steps: int = 0
+    rows_scored: int = 0
+
+
+def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float, mask_id: int,
+           hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
+           on_step: Callable | None = None) -> LoopStats:
+    """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
+
+    ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
+    for global step ``k``.  ``on_step(k, blk_start, counts_host, flags)`` is called
+    after every step (for tests and statistics).
+    """
+    import torch
+
+    n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
+    d, V = int(W.shape[1]), int(W.shape[0])
+    N = n_seq * 2 * blk_len
+    dev = tokens.device
+    ws = torch.zeros(wino_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
+    counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
+    flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
+    counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
+    stats = LoopStats()
+    k = 0
+    for b in range(n_blocks):
+        b0 = prompt_len + b * blk_len
+        p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps)
+        bs = BlockStats(block=b, blk_start=b0)
+        while True:
+            if bs.steps >= max_steps:
+                raise WinoError(WINO_ERR_MAX_STEPS, f"decode: block {b} not finished after {max_steps} steps")
+            H = hidden(k, b0)
+            wino_step(H, W, tokens, p, counts, ws, flags=flags, stream=stream)
+            counts_host.copy_(counts, non_blocking=True)
+            torch.cuda.current_stream(dev).synchronize() if stream is None else stream.synchronize()
+            c = counts_host.numpy()
+            if (c < 0).any():
+                raise WinoError(int(c.min()), f"decode: device status at step {k}")
+            bs.steps += 1
+            bs.drafted += int(c[:, 0].sum())
+            bs.remasked += int(c[:, 1].sum())
+            stats.rows_scored += N
+            if on_step is not None:
+                on_step(k, b0, c.copy(), flags)
+            k += 1
+            if (c[:, 2] == 0).all():
+                break
+        stats.blocks.append(bs)
+    stats.total_steps = k
+    return stats

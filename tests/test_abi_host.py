@@ -1,0 +1,109 @@
+"""The C ABI without a GPU: the library loads, exports every declared entry point,
+and rejects bad arguments before touching CUDA."""
+import ctypes as C
+import re
+from pathlib import Path
+
+import pytest
+
+import paper_2605_16941_gb300 as wino
+from paper_2605_16941_gb300 import _abi
+
+HEADER = Path(__file__).resolve().parents[1] / "include" / "wino.h"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2605_16941_gb300 import build
+    build.build()
+
+
+def declared_functions():
+    text = HEADER.read_text()
+    return re.findall(r"WINO_API\s+[\w\s\*]+?\b(wino_\w+)\s*\(", text)
+
+
+def test_every_declared_symbol_is_exported():
+    names = declared_functions()
+    assert set(names) == set(_abi.EXPORTS), names
+    L = C.CDLL(str(wino.library_path()))
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_status_strings_and_version():
+    assert wino.wino_version() == 1
+    for code in (0, -1, -2, -3, -4, -5, -6, -7):
+        assert wino.wino_status_string(code) != "unknown status"
+    assert wino.wino_status_string(12345) == "unknown status"
+
+
+def test_workspace_size():
+    n = wino.wino_workspace_size(256, 4096, 126464)
+    assert n >= 256 * 494 * 16 and n % 256 == 0
+    for bad in ((0, 64, 100), (64, 60, 100), (64, 4, 100), (64, 64, 1), (1 << 25, 64, 100), (64, 64, 1 << 28)):
+        with pytest.raises(wino.WinoError) as e:
+            wino.wino_workspace_size(*bad)
+        assert e.value.status == wino.WINO_ERR_SHAPE
+
+
+FAKE = 0x10000  # 16-byte (and 256-byte) aligned, never dereferenced: every call below fails its checks first
+
+
+def _p(**kw):
+    base = dict(tau1=0.7, tau2=0.9, mask_id=99, n_seq=2, seq_len=64, blk_start=32, blk_len=16, max_steps=10)
+    base.update(kw)
+    return _abi.WinoParams(*base.values())
+
+
+def test_score_rows_argument_errors():
+    L = wino.lib()
+    ok = dict(H=FAKE, W=FAKE, N=64, d=64, V=100, t=None, a=FAKE, pm=FAKE, pt=FAKE, ws=FAKE, wsb=1 << 20, s=None)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return L.wino_score_rows(a["H"], a["W"], a["N"], a["d"], a["V"], a["t"], a["a"], a["pm"], a["pt"], a["ws"],
+                                 a["wsb"], a["s"])
+    for k in ("H", "W", "a", "pm", "pt", "ws"):
+        assert call(**{k: None}) == wino.WINO_ERR_ARG, k
+    assert call(H=FAKE + 2) == wino.WINO_ERR_ARG
+    assert call(W=FAKE + 8) == wino.WINO_ERR_ARG
+    assert call(ws=FAKE + 16) == wino.WINO_ERR_ARG
+    assert call(d=60) == wino.WINO_ERR_SHAPE
+    assert call(N=0) == wino.WINO_ERR_SHAPE
+    assert call(V=1) == wino.WINO_ERR_SHAPE
+
+
+def test_draft_verify_argument_errors():
+    L = wino.lib()
+
+    def call(p, **kw):
+        a = dict(tok=FAKE, am=FAKE, pm=FAKE, pt=FAKE, cnt=FAKE)
+        a.update(kw)
+        return L.wino_draft_verify(a["tok"], a["am"], a["pm"], a["pt"], C.byref(p) if p is not None else None,
+                                   a["cnt"], None, None)
+    for k in ("tok", "am", "pm", "pt", "cnt"):
+        assert call(_p(), **{k: None}) == wino.WINO_ERR_ARG, k
+    assert call(None) == wino.WINO_ERR_ARG
+    assert call(_p(tau1=1.5)) == wino.WINO_ERR_ARG
+    assert call(_p(tau2=-0.1)) == wino.WINO_ERR_ARG
+    assert call(_p(tau1=float("nan"))) == wino.WINO_ERR_ARG
+    assert call(_p(blk_len=0)) == wino.WINO_ERR_SHAPE
+    assert call(_p(blk_len=1025, seq_len=2000)) == wino.WINO_ERR_SHAPE
+    assert call(_p(blk_start=50)) == wino.WINO_ERR_SHAPE  # block runs past seq_len
+    assert call(_p(n_seq=0)) == wino.WINO_ERR_SHAPE
+    assert call(_p(mask_id=-1)) == wino.WINO_ERR_SHAPE
+
+
+def test_step_argument_errors():
+    L = wino.lib()
+
+    def call(p, d=64, V=100, wsb=1 << 30, **kw):
+        a = dict(H=FAKE, W=FAKE, tok=FAKE, cnt=FAKE, ws=FAKE)
+        a.update(kw)
+        return L.wino_step(a["H"], a["W"], d, V, a["tok"], C.byref(p), a["cnt"], None, a["ws"], wsb, None)
+    for k in ("H", "W", "tok", "cnt", "ws"):
+        assert call(_p(), **{k: None}) == wino.WINO_ERR_ARG, k
+    assert call(_p(mask_id=100)) == wino.WINO_ERR_SHAPE  # MASK outside the vocabulary
+    assert call(_p(), d=12) == wino.WINO_ERR_SHAPE
+    assert call(_p(), wsb=1000) == wino.WINO_ERR_WORKSPACE

@@ -1,0 +1,252 @@
+"""GPU parity of wino_draft_verify / wino_step / the decode loop against the fp64 oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import wino_synth as ws
+
+pytestmark = pytest.mark.gpu
+
+
+def _random_case(rng, n_seq, L, S, b0, M):
+    tokens = rng.integers(0, M + 1, size=(n_seq, S)).astype(np.int32)
+    tokens[rng.random((n_seq, S)) < 0.4] = M
+    N = n_seq * 2 * L
+    am = rng.integers(0, M + 1, size=N).astype(np.int32)  # includes MASK itself now and then
+    pm = rng.random(N).astype(np.float32)
+    pt = rng.random(N).astype(np.float32)
+    pm[rng.random(N) < 0.05] = np.float32(0.5)  # exact threshold hits
+    pt[rng.random(N) < 0.05] = np.float32(0.75)
+    return tokens, am, pm, pt
+
+
+CASES = [(1, 1, 3, 1), (1, 32, 40, 4), (5, 31, 70, 2), (17, 33, 100, 50), (3, 128, 300, 100), (4, 256, 600, 0),
+         (2, 1024, 1030, 3)]
+
+
+@pytest.mark.parametrize("n_seq,L,S,b0", CASES, ids=[f"B{c[0]}_L{c[1]}" for c in CASES])
+@pytest.mark.parametrize("taus", [(0.5, 0.75), (0.7, 0.9), (1.0, 0.0), (0.0, 1.0)], ids=str)
+def test_draft_verify_bit_exact(n_seq, L, S, b0, taus):
+    """Given the same fp32 statistics, the kernel's Eq. 4 equals the oracle's bit for bit."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, f32, host
+    M = 997
+    rng = np.random.default_rng(n_seq * 1000 + L)
+    tokens, am, pm, pt = _random_case(rng, n_seq, L, S, b0, M)
+    t1, t2 = taus
+    ref_tok, ref_cnt, ref_fl = oracle.draft_verify(tokens, b0, L, M, f32(t1), f32(t2), am, pm.astype(np.float64),
+                                                   pt.astype(np.float64))
+    tok_d = dev(tokens)
+    counts = torch.full((n_seq, 3), -9, dtype=torch.int32, device="cuda")
+    flags = torch.full((n_seq, L), -9, dtype=torch.int8, device="cuda")
+    p = wino.make_params(t1, t2, M, n_seq, S, b0, L)
+    wino.wino_draft_verify(tok_d, dev(am), dev(pm), dev(pt), p, counts, flags)
+    torch.cuda.synchronize()
+    assert np.array_equal(host(tok_d), ref_tok)
+    assert np.array_equal(host(counts), ref_cnt)
+    assert np.array_equal(host(flags), ref_fl)
+
+
+def _gpu_step(w, Wd, tokens, H, blk_start, tau1=None):
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, host
+    tau1 = w.tau1 if tau1 is None else tau1
+    tok_d = dev(tokens)
+    counts = torch.full((w.n_seq, 3), -9, dtype=torch.int32, device="cuda")
+    flags = torch.full((w.n_seq, w.blk_len), -9, dtype=torch.int8, device="cuda")
+    ws_ = wino.workspace(w.N, w.d, w.V)
+    p = wino.make_params(tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, blk_start, w.blk_len)
+    wino.wino_step(dev(H), Wd, tok_d, p, counts, ws_, flags=flags)
+    torch.cuda.synchronize()
+    return host(tok_d), host(counts), host(flags)
+
+
+def _gpu_decomposed(w, Wd, tokens, H, blk_start, tau1):
+    """score_rows (targets from the oracle's gather) + draft_verify: the GPU's own statistics."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, gpu_score, host
+    t = oracle.row_targets(tokens, blk_start, w.blk_len, w.mask_id)
+    g = gpu_score(dev(H), Wd, t)
+    tok_d = dev(tokens)
+    counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device="cuda")
+    flags = torch.zeros((w.n_seq, w.blk_len), dtype=torch.int8, device="cuda")
+    p = wino.make_params(tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, blk_start, w.blk_len)
+    wino.wino_draft_verify(tok_d, dev(g.argmax), dev(g.pmax), dev(g.ptarget), p, counts, flags)
+    torch.cuda.synchronize()
+    return g, t, host(tok_d), host(counts), host(flags)
+
+
+def _check_full(w, W, Wd, tau1=None, step=0):
+    from gpu_helpers import compare_rows, compare_step
+    tau1 = w.tau1 if tau1 is None else tau1
+    st = ws.initial_state(w)
+    H = ws.hidden_states(w, W, st, step=step)
+    tok, cnt, fl = _gpu_step(w, Wd, st.tokens, H, st.blk_start, tau1)
+    o = oracle.step(H, W, st.tokens, st.blk_start, w.blk_len, w.mask_id, tau1, w.tau2)
+    rows = compare_rows(o, _gpu_decomposed(w, Wd, st.tokens, H, st.blk_start, tau1)[0])
+    rep = compare_step(st.tokens, tok, cnt, o, st.blk_start, w.blk_len, w.mask_id, tau1, w.tau2)
+    return rows, rep
+
+
+@pytest.mark.parametrize("variant", ["base", "coverage"])
+def test_step_tiny(variant):
+    from gpu_helpers import dev
+    w = ws.WORKLOADS["tiny"]
+    w = ws.coverage_variant(w) if variant == "coverage" else w
+    W = ws.weights(w)
+    Wd = dev(W)
+    for step in range(4):
+        rows, rep = _check_full(w, W, Wd, step=step)
+        print(f"tiny/{variant} step {step}: {rows} {rep}")
+
+
+@pytest.fixture(scope="module")
+def llada():
+    from gpu_helpers import dev
+    w = ws.WORKLOADS["llada_b1"]
+    W = ws.weights(w)
+    return W, dev(W)
+
+
+@pytest.mark.parametrize("variant", ["base", "coverage"])
+def test_step_llada_b1_full_oracle(llada, variant):
+    """N=256, d=4096, V=126464: the whole step against the whole oracle step."""
+    W, Wd = llada
+    w = ws.WORKLOADS["llada_b1"]
+    w = ws.coverage_variant(w) if variant == "coverage" else w
+    rows, rep = _check_full(w, W, Wd)
+    print(f"llada_b1/{variant}: {rows} {rep}")
+    if variant == "coverage":
+        assert rep["threshold_drafts"] > 0 and rep["kept_decoded"] > 0 and rep["remasked"] > 0
+
+
+def _check_sampled(w, W, Wd, tau1, n_rows=24):
+    """Full-size batch: every row's statistics sampled against the oracle; Eq. 4 exact on the GPU's
+    own statistics; wino_step identical to the decomposed path; invariants on every position."""
+    from gpu_helpers import compare_rows, f32
+    st = ws.initial_state(w)
+    H = ws.hidden_states(w, W, st, step=0)
+    tok, cnt, fl = _gpu_step(w, Wd, st.tokens, H, st.blk_start, tau1)
+    g, t, tok2, cnt2, fl2 = _gpu_decomposed(w, Wd, st.tokens, H, st.blk_start, tau1)
+    assert np.array_equal(tok, tok2) and np.array_equal(cnt, cnt2) and np.array_equal(fl, fl2)
+    ref_tok, ref_cnt, ref_fl = oracle.draft_verify(st.tokens, st.blk_start, w.blk_len, w.mask_id, f32(tau1),
+                                                   f32(w.tau2), g.argmax, g.pmax.astype(np.float64),
+                                                   g.ptarget.astype(np.float64))
+    assert np.array_equal(tok, ref_tok) and np.array_equal(cnt, ref_cnt) and np.array_equal(fl, ref_fl)
+    rows = np.random.default_rng(1).choice(w.N, n_rows, replace=False)
+    o = oracle.score_rows(H[rows], W, t[rows])
+    rep = compare_rows(o, g, rows)
+    L, b0 = w.blk_len, st.blk_start
+    pre = st.tokens[:, b0:b0 + L]
+    post = tok[:, b0:b0 + L]
+    assert np.array_equal(np.delete(tok, np.s_[b0:b0 + L], 1), np.delete(st.tokens, np.s_[b0:b0 + L], 1))
+    assert np.all((post == pre) | (pre == w.mask_id) | (post == w.mask_id))
+    return rep, {"drafted": int(cnt[:, 0].sum()), "remasked": int(cnt[:, 1].sum()), "left": int(cnt[:, 2].sum()),
+                 "fallback": int((fl == 2).sum())}
+
+
+@pytest.mark.parametrize("tau1", [0.5, 0.7, 0.9])
+def test_step_llada_b8_sampled(llada, tau1):
+    W, Wd = llada
+    w = ws.WORKLOADS["llada_b8"]
+    rep, c = _check_sampled(w, W, Wd, tau1)
+    print(f"llada_b8 tau1={tau1}: {rep} {c}")
+
+
+def test_step_unified_b4_sampled():
+    from gpu_helpers import dev
+    w = ws.WORKLOADS["unified_b4"]
+    W = ws.weights(w)
+    rep, c = _check_sampled(w, W, dev(W), w.tau1)
+    print(f"unified_b4: {rep} {c}")
+
+
+def test_decode_loop_tiny_lockstep():
+    """The tiny workload decoded to the end through the package's loop driver; every step is
+    re-run by the oracle from the same pre-step state and compared."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import compare_step, dev, host
+    w = ws.Workload("tiny_loop", d=64, V=1000, n_seq=2, blk_len=32, bias=((1.0, 0.0, 6.0),), n_blocks=3,
+                    bias_step=0.5, tau1=0.7, tau2=0.9)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    tok_d = dev(st.tokens)
+    record = {}
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        H = ws.hidden_states(w, W, st, step=k)
+        record["pre"] = host(tok_d).copy()
+        record["H"] = H
+        return dev(H)
+
+    reports = []
+
+    def on_step(k, b0, counts, flags):
+        o = oracle.step(record["H"], W, record["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2)
+        reports.append(compare_step(record["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1,
+                                    w.tau2))
+
+    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=500)
+    final = host(tok_d)
+    assert not np.any(final[:, w.prompt_len:] == w.mask_id)
+    assert np.array_equal(final[:, :w.prompt_len], st.tokens[:, :w.prompt_len])
+    print("tiny loop steps/block", [b.steps for b in stats.blocks], "flagged",
+          sum(r["flagged_positions"] for r in reports))
+
+
+def test_decode_loop_b16():
+    """Config-5 loop (B=16, gen 256 in 8 blocks of 32, bias U[0, 4 + 0.5 k] at global step k):
+    runs until no MASK remains; invariants on every step; the oracle re-checks sampled steps."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import compare_rows, dev, f32, gpu_score, host
+    w = ws.WORKLOADS["loop_b16"]
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    tok_d = dev(st.tokens)
+    rec = {}
+    sampled = {0, 1, 2, 3, 40, 200}
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        H = ws.hidden_states(w, W, st, step=k)
+        rec["pre"] = host(tok_d).copy()
+        rec["H"] = H
+        rec["Hd"] = dev(H)
+        return rec["Hd"]
+
+    checked = []
+
+    def on_step(k, b0, counts, flags):
+        pre, post = rec["pre"], host(tok_d)
+        L = w.blk_len
+        outside = np.ones(w.seq_len, bool)
+        outside[b0:b0 + L] = False
+        assert np.array_equal(post[:, outside], pre[:, outside])
+        a, b = pre[:, b0:b0 + L], post[:, b0:b0 + L]
+        fl = host(flags)
+        assert np.all((b == a) | (a == w.mask_id) | (b == w.mask_id))
+        had_mask = (a == w.mask_id).any(1)
+        assert np.all((counts[:, 0] >= 1) | ~had_mask | (fl == 4).any(1))
+        assert np.array_equal(counts[:, 2], (b == w.mask_id).sum(1))
+        if k in sampled:
+            t = oracle.row_targets(pre, b0, L, w.mask_id)
+            g = gpu_score(rec["Hd"], Wd, t)
+            ref = oracle.draft_verify(pre, b0, L, w.mask_id, f32(w.tau1), f32(w.tau2), g.argmax,
+                                      g.pmax.astype(np.float64), g.ptarget.astype(np.float64))
+            assert np.array_equal(post, ref[0]) and np.array_equal(counts, ref[1])
+            rows = np.random.default_rng(k).choice(w.N, 8, replace=False)
+            compare_rows(oracle.score_rows(rec["H"][rows], W, t[rows]), g, rows)
+            checked.append(k)
+
+    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=4096)
+    final = host(tok_d)
+    assert not np.any(final[:, w.prompt_len:] == w.mask_id)
+    print("loop_b16 steps/block", [b.steps for b in stats.blocks], "total", stats.total_steps,
+          "drafted/block", [b.drafted for b in stats.blocks], "remasked/block", [b.remasked for b in stats.blocks],
+          "oracle-checked steps", checked)

@@ -33,7 +33,8 @@ MUTANTS = [
     ("softmax_sign_flip", "Z += exp(logit[v] - m);", "Z += exp(m - logit[v]);"),
     ("pmax_not_inverted", "pmax[n] = 1.0 / Z;", "pmax[n] = Z / V;"),
     ("ptarget_uses_argmax", "exp(logit[t] - m) / Z", "exp(logit[a] - m) / Z"),
-    ("hidden_index_reversed", "oracle_bf16_to_double(h[k]) *", "oracle_bf16_to_double(h[d - 1 - k]) *"),
+    ("hidden_index_reversed", "hd[k] = oracle_bf16_to_double(h[k]);", "hd[k] = oracle_bf16_to_double(h[d - 1 - k]);"),
+    ("weight_row_stride_wrong", "const uint16_t *w = W + v * d;", "const uint16_t *w = W + v;"),
     ("bf16_wrong_shift", "(uint32_t)bits << 16;", "(uint32_t)bits << 15;"),
     ("verify_target_on_block_row", "target[(s * 2 + 1) * blk_len + l] = (y == mask_id) ? -1 : y;",
      "target[(s * 2 + 0) * blk_len + l] = (y == mask_id) ? -1 : y;"),
