@@ -67,7 +67,17 @@ typedef struct {
     int32_t blk_start; /* first position of the current block Y_cur                             */
     int32_t blk_len;   /* L_b, 1..1024; blk_start + blk_len <= seq_len                           */
     int32_t max_steps; /* step budget for loop drivers; unused by the calls below               */
+    int32_t options;   /* bit set of WINO_OPT_* below; 0 = plain Eq. 4 on every sequence        */
 } wino_params;
+
+/*
+ * WINO_OPT_FREEZE_FINISHED: a sequence whose current block holds no MASK
+ * before the step is finished -- the per-sequence loop of Sec. 4.2.3 stops
+ * there -- and is left unchanged (counts {0, 0, 0}, flags 0).  Batched decode
+ * loops set it so that sequences that finish early are not re-verified while
+ * they wait for the rest of the batch.
+ */
+#define WINO_OPT_FREEZE_FINISHED 1
 
 /*
  * Bytes of scratch the score path needs for N rows of dimension d over a

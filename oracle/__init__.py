@@ -64,10 +64,10 @@ class Oracle:
         L.oracle_row_targets.restype = C.c_int
         L.oracle_row_targets.argtypes = [vp, i64, i64, i64, i64, i32, vp]
         L.oracle_draft_verify.restype = C.c_int
-        L.oracle_draft_verify.argtypes = [vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp]
+        L.oracle_draft_verify.argtypes = [vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp, C.c_int]
         L.oracle_step.restype = C.c_int
         L.oracle_step.argtypes = [vp, vp, i64, i64, vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp,
-                                  vp, C.c_int]
+                                  vp, C.c_int, C.c_int]
         L.oracle_num_threads.restype = C.c_int
         L.oracle_num_threads.argtypes = []
         self.L = L
@@ -113,7 +113,8 @@ class Oracle:
         return out
 
     def draft_verify(self, tokens: np.ndarray, blk_start: int, blk_len: int, mask_id: int, tau1: float,
-                     tau2: float, argmax: np.ndarray, pmax: np.ndarray, ptarget: np.ndarray):
+                     tau2: float, argmax: np.ndarray, pmax: np.ndarray, ptarget: np.ndarray,
+                     freeze_finished: bool = False):
         """Eq. 4 on a copy of ``tokens``; returns (new_tokens, counts [n_seq,3], flags [n_seq, blk_len])."""
         tok = np.array(tokens, dtype=np.int32, copy=True, order="C")
         n_seq, S = tok.shape
@@ -123,13 +124,14 @@ class Oracle:
         counts = np.empty((n_seq, 3), np.int32)
         flags = np.empty((n_seq, blk_len), np.int8)
         rc = self.L.oracle_draft_verify(_p(tok), n_seq, S, blk_start, blk_len, mask_id, float(tau1),
-                                        float(tau2), _p(am), _p(pm), _p(pt), _p(counts), _p(flags))
+                                        float(tau2), _p(am), _p(pm), _p(pt), _p(counts), _p(flags),
+                                        int(bool(freeze_finished)))
         if rc != 0:
             raise RuntimeError(f"oracle_draft_verify failed: {rc}")
         return tok, counts, flags
 
     def step(self, H_bits: np.ndarray, W_bits: np.ndarray, tokens: np.ndarray, blk_start: int, blk_len: int,
-             mask_id: int, tau1: float, tau2: float, nthreads: int = 0) -> StepResult:
+             mask_id: int, tau1: float, tau2: float, nthreads: int = 0, freeze_finished: bool = False) -> StepResult:
         """One whole WINO step on a copy of ``tokens``."""
         H, W = _c(H_bits, np.uint16), _c(W_bits, np.uint16)
         tok = np.array(tokens, dtype=np.int32, copy=True, order="C")
@@ -142,7 +144,7 @@ class Oracle:
                        np.empty(N, np.float64))
         rc = self.L.oracle_step(_p(H), _p(W), d, V, _p(tok), n_seq, S, blk_start, blk_len, mask_id, float(tau1),
                                 float(tau2), _p(r.counts), _p(r.flags), _p(r.argmax), _p(r.pmax), _p(r.ptarget),
-                                _p(r.gap), nthreads)
+                                _p(r.gap), nthreads, int(bool(freeze_finished)))
         if rc != 0:
             raise RuntimeError(f"oracle_step failed: {rc}")
         return r
@@ -178,9 +180,11 @@ def row_targets(tokens, blk_start: int, blk_len: int, mask_id: int):
     return default().row_targets(tokens, blk_start, blk_len, mask_id)
 
 
-def draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget):
-    return default().draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget)
+def draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget, freeze_finished=False):
+    return default().draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget,
+                                  freeze_finished)
 
 
-def step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads: int = 0) -> StepResult:
-    return default().step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads)
+def step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads: int = 0,
+         freeze_finished: bool = False) -> StepResult:
+    return default().step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads, freeze_finished)

@@ -175,11 +175,14 @@ int oracle_row_targets(const int32_t *tokens, int64_t n_seq, int64_t seq_len, in
  * Both conditions read y^(k-1), so D and R are disjoint and the update is
  * simultaneous.  counts[s] = {drafted (MASK -> token), re-masked, MASKs left
  * in the block}; flags[s * blk_len + l] (optional) gets the outcome codes.
+ * With freeze_finished != 0, a sequence whose block has no MASK is not
+ * stepped at all: the loop "until no MASK is left" (Sec. 4.2.3) has ended
+ * for it.
  */
 int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t blk_start,
                         int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                         const int32_t *argmax, const double *pmax, const double *ptarget,
-                        int32_t *counts, int8_t *flags)
+                        int32_t *counts, int8_t *flags, int freeze_finished)
 {
     if (!tokens || !argmax || !pmax || !ptarget || !counts || n_seq < 0 || blk_len < 1 ||
         blk_start < 0 || blk_start + blk_len > seq_len)
@@ -204,6 +207,13 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
             inR[l] = (prev[l] != mask_id) && (ptarget[row_shd + l] < tau2);
             n_draft += inD[l];
             n_mask += (prev[l] == mask_id);
+        }
+        if (freeze_finished && n_mask == 0) {
+            for (int64_t l = 0; l < blk_len; ++l)
+                if (flags)
+                    flags[s * blk_len + l] = 0;
+            counts[s * 3 + 0] = counts[s * 3 + 1] = counts[s * 3 + 2] = 0;
+            continue;
         }
         int64_t fallback = -1;
         if (n_draft == 0 && n_mask > 0) {
@@ -254,7 +264,7 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
 int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, int64_t n_seq,
                 int64_t seq_len, int64_t blk_start, int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                 int32_t *counts, int8_t *flags, int32_t *argmax_out, double *pmax_out, double *ptarget_out,
-                double *gap_out, int nthreads)
+                double *gap_out, int nthreads, int freeze_finished)
 {
     const int64_t N = n_seq * 2 * blk_len;
     int32_t *target = (int32_t *)malloc((size_t)N * sizeof(int32_t));
@@ -269,7 +279,7 @@ int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int3
             rc = oracle_score_rows(H, W, N, d, V, target, am, pm, pt, gp, NULL, NULL, nthreads);
         if (rc == ORACLE_OK)
             rc = oracle_draft_verify(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, tau1, tau2, am, pm,
-                                     pt, counts, flags);
+                                     pt, counts, flags, freeze_finished);
         if (rc == ORACLE_OK) {
             if (argmax_out)
                 memcpy(argmax_out, am, (size_t)N * sizeof(int32_t));

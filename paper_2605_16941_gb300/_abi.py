@@ -26,6 +26,9 @@ WINO_ERR_UNSUPPORTED = -7
 # per-position outcome codes written to `flags`
 FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0, 1, 2, 3, 4
 
+# wino_params.options
+WINO_OPT_FREEZE_FINISHED = 1
+
 EXPORTS = ("wino_workspace_size", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_read_device_status", "wino_profile_begin", "wino_profile_end", "wino_status_string",
            "wino_version")
@@ -40,7 +43,7 @@ class WinoError(RuntimeError):
 class WinoParams(C.Structure):
     _fields_ = [("tau1", C.c_float), ("tau2", C.c_float), ("mask_id", C.c_int32), ("n_seq", C.c_int32),
                 ("seq_len", C.c_int32), ("blk_start", C.c_int32), ("blk_len", C.c_int32),
-                ("max_steps", C.c_int32)]
+                ("max_steps", C.c_int32), ("options", C.c_int32)]
 
 
 def library_path() -> Path:
@@ -120,8 +123,9 @@ def workspace(N: int, d: int, V: int, device=None):
 
 
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
-                max_steps: int = 4096) -> WinoParams:
-    return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps)
+                max_steps: int = 4096, freeze_finished: bool = False) -> WinoParams:
+    return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps,
+                      WINO_OPT_FREEZE_FINISHED if freeze_finished else 0)
 
 
 def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, N: int | None = None,

@@ -1,0 +1,238 @@
+// finish.cu -- the end of a WINO step (sm_103a): merge the score kernel's
+// partial softmax records per row, then apply Eq. 4 to the token state.
+//
+// finish_kernel: one warp per row folds the row's G partial records (fixed
+// lane order, then a butterfly, so results are bit-for-bit reproducible) into
+//   argmax   = smallest vocabulary id among the maximal logits,
+//   pmax     = max_v p_v = 1 / sum_v exp(l_v - m),
+//   ptarget  = p_target = exp(l_t - m) / sum_v exp(l_v - m)    (0 without a target),
+// the three statistics Eq. 2 and Eq. 3 use.  In a whole step (wino_step) every
+// CTA then adds its merged rows to its sequences' tickets; the CTA that
+// completes a sequence's 2*L_b rows applies Eq. 4 to that sequence, so merge
+// and update need one launch.  Tickets are cleared by the score kernel of the
+// same step.  The kernel is launched programmatically: its launch overlaps the
+// score kernel and it waits (griddepcontrol.wait) for the score kernel's
+// results before touching them.
+//
+// draft_verify_kernel: Eq. 4 alone from caller-supplied statistics
+// (wino_draft_verify).
+//
+// Eq. 4, per sequence, reading the state before the step y^(k-1):
+//   draft  (Eq. 2): y_l == MASK and pmax(block row l) > tau1      -> argmax(block row l)
+//   verify (Eq. 3): y_l != MASK and p(y_l | shadow row l) < tau2  -> MASK
+// and, if no masked position clears tau1 while the block still has a MASK,
+// the masked position with the largest pmax (smallest position on ties) is
+// drafted: the greedy rule of Eq. 1, which keeps at least one token coming per
+// step.  The rules touch disjoint positions (MASK vs not MASK), so the update
+// is applied in place in one pass after a warp-wide reduction.  With
+// WINO_OPT_FREEZE_FINISHED a sequence whose block already has no MASK is left
+// as it is (its own loop, Sec. 4.2.3, has ended).
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace wino {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kFinishRows = 8;  // rows (warps) per finish CTA
+constexpr int kDVWarps = 4;     // sequences (warps) per draft_verify CTA
+
+// Fold (m2, s2, i2) into (m, s, i): the larger max wins, the smaller index on equal maxima.
+__device__ __forceinline__ void combine(float &m, float &s, int32_t &i, float m2, float s2, int32_t i2)
+{
+    const float M = fmaxf(m, m2);
+    const float a = (m == -INFINITY) ? 0.f : s * ptx::ex2((m - M) * kLog2e);
+    const float b = (m2 == -INFINITY) ? 0.f : s2 * ptx::ex2((m2 - M) * kLog2e);
+    if (m2 > m || (m2 == m && i2 < i))
+        i = i2;
+    m = M;
+    s = a + b;
+}
+
+// Eq. 4 on sequence s by one warp.  Statistics are read through L2 (other CTAs may have written them).
+__device__ void eq4_sequence(int s, int lane, int32_t *tokens, const int32_t *argmax, const float *pmax,
+                             const float *ptarget, const wino_params &p, int32_t *counts, int8_t *flags,
+                             int32_t status)
+{
+    if (status != WINO_OK) {  // the scores of this step are invalid: leave the state alone
+        if (lane < 3)
+            counts[s * 3 + lane] = status;
+        return;
+    }
+    const int L = p.blk_len;
+    const int32_t mask = p.mask_id;
+    int32_t *y = tokens + (int64_t)s * p.seq_len + p.blk_start;
+    const int64_t rb = (int64_t)(2 * s) * L;      // kind-0 rows: the block Y_cur
+    const int64_t rs = (int64_t)(2 * s + 1) * L;  // kind-1 rows: the shadow block Y_shad
+
+    // Pass 1: how many masked positions clear tau1, and the most confident masked position.
+    int n_clear = 0, n_mask = 0;
+    float best = -INFINITY;
+    int best_l = INT32_MAX;
+    for (int l = lane; l < L; l += 32) {
+        if (y[l] == mask) {
+            const float pm = __ldcg(pmax + rb + l);
+            ++n_mask;
+            n_clear += (pm > p.tau1);
+            if (pm > best || (pm == best && l < best_l)) {
+                best = pm;
+                best_l = l;
+            }
+        }
+    }
+    n_clear = __reduce_add_sync(0xffffffffu, n_clear);
+    n_mask = __reduce_add_sync(0xffffffffu, n_mask);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float b2 = __shfl_xor_sync(0xffffffffu, best, off);
+        const int l2 = __shfl_xor_sync(0xffffffffu, best_l, off);
+        if (b2 > best || (b2 == best && l2 < best_l)) {
+            best = b2;
+            best_l = l2;
+        }
+    }
+    if (n_mask == 0 && (p.options & WINO_OPT_FREEZE_FINISHED)) {  // finished block: its loop has stopped
+        if (flags)
+            for (int l = lane; l < L; l += 32)
+                flags[(int64_t)s * L + l] = 0;
+        if (lane < 3)
+            counts[s * 3 + lane] = 0;
+        return;
+    }
+    const int fallback = (n_clear == 0 && n_mask > 0) ? best_l : -1;
+
+    // Pass 2: apply Eq. 4 simultaneously.
+    int drafted = 0, remasked = 0, left = 0;
+    for (int l = lane; l < L; l += 32) {
+        const int32_t prev = y[l];
+        int32_t next = prev;
+        int8_t code = 0;
+        if (prev == mask) {
+            if (__ldcg(pmax + rb + l) > p.tau1 || l == fallback) {
+                next = __ldcg(argmax + rb + l);
+                code = (next == mask) ? 4 : (l == fallback ? 2 : 1);
+            }
+        } else if (__ldcg(ptarget + rs + l) < p.tau2) {
+            next = mask;
+            code = 3;
+        }
+        if (next != prev)
+            y[l] = next;
+        drafted += (code == 1 || code == 2);
+        remasked += (code == 3);
+        left += (next == mask);
+        if (flags)
+            flags[(int64_t)s * L + l] = code;
+    }
+    drafted = __reduce_add_sync(0xffffffffu, drafted);
+    remasked = __reduce_add_sync(0xffffffffu, remasked);
+    left = __reduce_add_sync(0xffffffffu, left);
+    if (lane == 0) {
+        counts[s * 3 + 0] = drafted;
+        counts[s * 3 + 1] = remasked;
+        counts[s * 3 + 2] = left;
+    }
+}
+
+__global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishArgs a)
+{
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch_dependents();
+    __shared__ int32_t s_done[kFinishRows];
+    __shared__ int32_t s_ndone;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t row0 = (int64_t)blockIdx.x * kFinishRows;
+    const int64_t row = row0 + warp;
+    const int32_t status = a.status ? *a.status : WINO_OK;
+
+    if (row < a.N) {
+        if (status != WINO_OK) {
+            if (lane == 0) {
+                a.argmax[row] = -1;
+                a.pmax[row] = __int_as_float(0x7fc00000);
+                a.ptarget[row] = __int_as_float(0x7fc00000);
+            }
+        } else {
+            const float4 *pr = a.part + row * a.G;
+            float m = -INFINITY, s = 0.f;
+            int32_t idx = INT32_MAX;
+            for (int j = lane; j < a.G; j += 32) {
+                const float4 r = __ldcg(pr + j);
+                combine(m, s, idx, r.x, r.y, __float_as_int(r.z));
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+                const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+                const int32_t i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+                combine(m, s, idx, m2, s2, i2);
+            }
+            if (lane == 0) {
+                const int32_t t = row_target(a.ts, row, a.V);
+                a.argmax[row] = idx;
+                a.pmax[row] = 1.0f / s;
+                a.ptarget[row] = (t >= 0) ? ptx::ex2((__ldcg(pr + (t / kBN) % a.G).w - m) * kLog2e) / s : 0.0f;
+                __threadfence();  // publish this row before the CTA signals its ticket
+            }
+        }
+    }
+    if (!a.tokens)
+        return;
+
+    // Eq. 4: the CTA that merges the last rows of a sequence updates that sequence.
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t nd = 0;
+        const int64_t per_seq = 2 * (int64_t)a.p.blk_len;
+        const int64_t rend = min(row0 + kFinishRows, (int64_t)a.N);
+        for (int64_t r = row0; r < rend;) {
+            const int64_t sq = r / per_seq;
+            const int64_t send = min((sq + 1) * per_seq, rend);
+            const int32_t cnt = (int32_t)(send - r);
+            if (atomicAdd(&a.tickets[sq], cnt) + cnt == per_seq)
+                s_done[nd++] = (int32_t)sq;
+            r = send;
+        }
+        s_ndone = nd;
+        __threadfence();
+    }
+    __syncthreads();
+    for (int i = warp; i < s_ndone; i += kFinishRows)
+        eq4_sequence(s_done[i], lane, a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status);
+}
+
+__global__ void __launch_bounds__(kDVWarps * 32)
+    draft_verify_kernel(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
+                        const wino_params p, int32_t *counts, int8_t *flags)
+{
+    const int s = blockIdx.x * kDVWarps + (threadIdx.x >> 5);
+    if (s < p.n_seq)
+        eq4_sequence(s, threadIdx.x & 31, tokens, argmax, pmax, ptarget, p, counts, flags, WINO_OK);
+}
+
+}  // namespace
+
+cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((a.N + kFinishRows - 1) / kFinishRows));
+    cfg.blockDim = dim3(kFinishRows * 32);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, finish_kernel, a);
+}
+
+cudaError_t launch_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
+                                const wino_params &p, int32_t *counts, int8_t *flags, cudaStream_t stream)
+{
+    const int blocks = (p.n_seq + kDVWarps - 1) / kDVWarps;
+    draft_verify_kernel<<<blocks, kDVWarps * 32, 0, stream>>>(tokens, argmax, pmax, ptarget, p, counts, flags);
+    return cudaGetLastError();
+}
+
+}  // namespace wino

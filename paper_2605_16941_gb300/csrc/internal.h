@@ -51,26 +51,51 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
     return (t >= 0 && t < V) ? t : -1;
 }
 
-// One partial softmax record per (row, vocabulary tile): running max logit m,
-// sum of exp(l - m) over the tile, argmax (int bits) and the target's logit
-// when the target lies in the tile (else 0).  Layout [row][tile].
+// Work split of the score kernel.  The row blocks are spread over n_groups
+// groups of G CTAs; CTA c serves row blocks c % n_groups (+ n_groups, ...) and,
+// within each, vocabulary tiles c / n_groups (+ G, ...).  The G CTAs of a group
+// walk the vocabulary side by side, so all groups read the same W tiles at the
+// same time (W streams from HBM about once), and each CTA keeps its running
+// softmax state per row across its tiles and writes ONE partial record per
+// (row, CTA of the group): G records per row.
+constexpr int kMaxRecordsPerRow = 256;
+
+// Partial record: running max logit m, sum of exp(l - m), argmax (int bits),
+// logit of the row's target if the target lies in one of the CTA's tiles (else 0).
 struct ScoreArgs {
     int32_t N, d, V;
     int32_t n_mb, n_vt, n_kb;
-    int64_t n_tiles;
+    int32_t n_groups, G;
     TargetSource ts;
-    float4 *part;
-    int32_t *status;
+    float4 *part;       // [N][G]
+    int32_t *status;    // cleared by CTA 0
+    int32_t *tickets;   // [n_tickets], cleared here for the finish kernel
+    int32_t n_tickets;
 };
 
-cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, int grid,
-                         cudaStream_t stream);
+struct FinishArgs {
+    const float4 *part;
+    int32_t G, N, V;
+    TargetSource ts;
+    const int32_t *status;
+    int32_t *argmax;
+    float *pmax;
+    float *ptarget;
+    // Eq. 4 in the same launch when tokens != nullptr (wino_step)
+    int32_t *tokens;
+    wino_params p;
+    int32_t *counts;
+    int8_t *flags;
+    int32_t *tickets;  // [n_seq], zero on entry
+};
 
-cudaError_t launch_merge(const float4 *part, int32_t N, int32_t n_vt, int32_t V, const TargetSource &ts,
-                         const int32_t *status, int32_t *argmax, float *pmax, float *ptarget, cudaStream_t stream);
+void score_schedule(int32_t n_mb, int32_t n_vt, int max_ctas, int32_t *n_groups, int32_t *G);
+
+cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream);
+
+cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream);
 
 cudaError_t launch_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
-                                const wino_params &p, int32_t *counts, int8_t *flags, const int32_t *status,
-                                cudaStream_t stream);
+                                const wino_params &p, int32_t *counts, int8_t *flags, cudaStream_t stream);
 
 }  // namespace wino

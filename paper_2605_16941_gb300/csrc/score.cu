@@ -3,30 +3,28 @@
 // For every scored row h_n the method needs three numbers of the model's
 // distribution p(. | Y~) = softmax_v(<h_n, w_v>) over the whole vocabulary
 // (Eq. 2 and Eq. 3 of the WINO paper): argmax_v p, max_v p and p(target).
-// The logits never leave the chip: each CTA computes a 128 x 256 logit tile
+// The logits never leave the chip: each CTA computes 128 x 256 logit tiles
 // on the tensor cores (tcgen05.mma, bf16 x bf16 -> fp32 in TMEM), and four
-// epilogue warps reduce it straight out of TMEM into a per-(row, tile) partial
-// record (max, sum of exp, argmax, target logit).  `merge_kernel` then folds
-// the records of a row across vocabulary tiles.
+// epilogue warps fold each tile straight out of TMEM into a running
+// per-row state (max, sum of exp, argmax, target logit) that lives in
+// registers across all of the CTA's vocabulary tiles of that row block.  One
+// partial record per (row, CTA) goes to the workspace; finish.cu merges them.
 //
 // Kernel structure (persistent, one CTA per SM, 192 threads):
 //   warp 0  TMA producer: streams 64-wide K slices of H (128 rows) and W
 //           (256 vocabulary rows) into a 4-stage shared-memory ring;
 //   warp 1  MMA issuer: allocates 512 TMEM columns (two 256-column fp32
 //           accumulators), issues 4 x (M128 N256 K16) MMAs per stage and
-//           commits stage release / accumulator-ready barriers;
+//           commits stage-release / accumulator-ready barriers;
 //   warps 2-5 epilogue: one thread per row (TMEM lane), online softmax over
-//           the tile's 256 columns while the MMA warp fills the other
+//           each tile's 256 columns while the MMA warp fills the other
 //           accumulator.
-// Tiles are ordered vocabulary-major (tile t -> row block t % n_mb, vocab
-// tile t / n_mb) so that the CTAs working at one time share W tiles in L2 and
-// W is streamed from HBM about once.
+// Work split: see ScoreArgs in internal.h (row-block groups walking the
+// vocabulary side by side).
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA raises an
 // abort flag, records WINO_ERR_DEVICE_TIMEOUT in the status word, drains its
 // in-flight copies and MMAs (again bounded) and frees its TMEM.
-#include <cfloat>
-
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -97,8 +95,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     auto tfull = [&](int s) { return ptx::smem_u32(&bars->tmem_full[s]); };
     auto tempty = [&](int s) { return ptx::smem_u32(&bars->tmem_empty[s]); };
 
-    if (blockIdx.x == 0 && threadIdx.x == 0)
-        *a.status = WINO_OK;  // a timeout, if any, is raised no earlier than kWaitLimitNs later
+    // Set-up that touches no global memory overlaps the previous kernel (programmatic launch).
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(full(s), 1);
@@ -125,37 +122,49 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     ptx::tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
 
+    // From here on global memory is read and written: wait for the grid before us.
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch_dependents();
+    if (blockIdx.x == 0 && threadIdx.x == 0)
+        *a.status = WINO_OK;  // a timeout, if any, is raised no earlier than kWaitLimitNs later
+    for (int i = blockIdx.x * kScoreThreads + threadIdx.x; i < a.n_tickets; i += gridDim.x * kScoreThreads)
+        a.tickets[i] = 0;
+
+    const int grp = blockIdx.x % a.n_groups;  // row blocks grp, grp + n_groups, ...
+    const int col = blockIdx.x / a.n_groups;  // vocabulary tiles col, col + G, ...
+
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
-        const uint64_t pol_h = ptx::policy_evict_last();   // H is re-read for every vocabulary tile
-        const uint64_t pol_w = ptx::policy_evict_normal(); // W is shared by the row blocks of one tile
+        const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every vocabulary tile
+        const uint64_t pol_w = ptx::policy_evict_normal();  // W is shared by the row-block groups
         int stage = 0;
         uint32_t phase = 0;
         int32_t issued_parity[kStages];
         for (int s = 0; s < kStages; ++s)
             issued_parity[s] = -1;
         bool aborted = false;
-        for (int64_t t = blockIdx.x; t < a.n_tiles && !aborted; t += gridDim.x) {
-            const int mb = (int)(t % a.n_mb), vt = (int)(t / a.n_mb);
-            for (int kb = 0; kb < a.n_kb; ++kb) {
-                int ok = 1;
-                if (lane == 0)
-                    ok = wait_bounded(empty(stage), phase ^ 1u, &bars->abort, a.status);
-                ok = __shfl_sync(0xffffffffu, ok, 0);
-                if (!ok) {
-                    aborted = true;
-                    break;
-                }
-                if (lane == 0) {
-                    ptx::mbar_arrive_expect_tx(full(stage), kStageBytesA + kStageBytesB);
-                    ptx::tma_load_2d(sA(stage), &tmH, full(stage), kb * kBK, mb * kBM, pol_h);
-                    ptx::tma_load_2d(sB(stage), &tmW, full(stage), kb * kBK, vt * kBN, pol_w);
-                }
-                __syncwarp();
-                issued_parity[stage] = (int32_t)phase;
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1u;
+        for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
+            for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
+                for (int kb = 0; kb < a.n_kb; ++kb) {
+                    int ok = 1;
+                    if (lane == 0)
+                        ok = wait_bounded(empty(stage), phase ^ 1u, &bars->abort, a.status);
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (!ok) {
+                        aborted = true;
+                        break;
+                    }
+                    if (lane == 0) {
+                        ptx::mbar_arrive_expect_tx(full(stage), kStageBytesA + kStageBytesB);
+                        ptx::tma_load_2d(sA(stage), &tmH, full(stage), kb * kBK, mb * kBM, pol_h);
+                        ptx::tma_load_2d(sB(stage), &tmW, full(stage), kb * kBK, vt * kBN, pol_w);
+                    }
+                    __syncwarp();
+                    issued_parity[stage] = (int32_t)phase;
+                    if (++stage == kStages) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
                 }
             }
         }
@@ -174,49 +183,51 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         bool aborted = false;
-        for (int64_t t = blockIdx.x; t < a.n_tiles && !aborted; t += gridDim.x) {
-            int ok = 1;
-            if (lane == 0)
-                ok = wait_bounded(tempty(acc), acc_phase ^ 1u, &bars->abort, a.status);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) {
-                aborted = true;
-                break;
-            }
-            ptx::tc_fence_after();
-            const uint32_t d_tmem = tmem + (uint32_t)(acc * kBN);
-            for (int kb = 0; kb < a.n_kb; ++kb) {
-                ok = 1;
+        for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
+            for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
+                int ok = 1;
                 if (lane == 0)
-                    ok = wait_bounded(full(stage), phase, &bars->abort, a.status);
+                    ok = wait_bounded(tempty(acc), acc_phase ^ 1u, &bars->abort, a.status);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) {
                     aborted = true;
                     break;
                 }
                 ptx::tc_fence_after();
-                if (lane == 0) {
-                    const uint64_t da = ptx::sdesc_kmajor_sw128(sA(stage));
-                    const uint64_t db = ptx::sdesc_kmajor_sw128(sB(stage));
+                const uint32_t d_tmem = tmem + (uint32_t)(acc * kBN);
+                for (int kb = 0; kb < a.n_kb; ++kb) {
+                    ok = 1;
+                    if (lane == 0)
+                        ok = wait_bounded(full(stage), phase, &bars->abort, a.status);
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (!ok) {
+                        aborted = true;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    if (lane == 0) {
+                        const uint64_t da = ptx::sdesc_kmajor_sw128(sA(stage));
+                        const uint64_t db = ptx::sdesc_kmajor_sw128(sB(stage));
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
-                        ptx::mma_bf16(d_tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
-                    ptx::mma_commit(empty(stage));
+                        for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
+                            ptx::mma_bf16(d_tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
+                        ptx::mma_commit(empty(stage));
+                    }
+                    __syncwarp();
+                    if (++stage == kStages) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
                 }
+                if (aborted)
+                    break;
+                if (lane == 0)
+                    ptx::mma_commit(tfull(acc));
                 __syncwarp();
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1u;
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
                 }
-            }
-            if (aborted)
-                break;
-            if (lane == 0)
-                ptx::mma_commit(tfull(acc));
-            __syncwarp();
-            if (++acc == 2) {
-                acc = 0;
-                acc_phase ^= 1u;
             }
         }
         // No MMA may still be writing TMEM when it is released.
@@ -230,82 +241,84 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         const int q = warp & 3;  // this warp may only read TMEM lanes [32q, 32q + 32)
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int64_t t = blockIdx.x; t < a.n_tiles; t += gridDim.x) {
-            const int mb = (int)(t % a.n_mb), vt = (int)(t / a.n_mb);
+        bool aborted = false;
+        for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
             const int64_t row = (int64_t)mb * kBM + q * 32 + lane;
-            const int32_t v0 = vt * kBN;
-            const int nvalid = min(kBN, a.V - v0);
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
-
-            int ok = 1;
-            if (lane == 0)
-                ok = wait_bounded(tfull(acc), acc_phase, &bars->abort, a.status);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok)
-                break;
-            ptx::tc_fence_after();
-            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
-
             float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tl = 0.f;
-            int32_t am = v0;
-#pragma unroll 1
-            for (int c = 0; c < kBN / 32; ++c) {
-                const int cvalid = nvalid - c * 32;  // warp-uniform
-                if (cvalid <= 0)
+            int32_t am = 0;
+            for (int vt = col; vt < a.n_vt; vt += a.G) {
+                const int32_t v0 = vt * kBN;
+                const int nvalid = min(kBN, a.V - v0);
+                int ok = 1;
+                if (lane == 0)
+                    ok = wait_bounded(tfull(acc), acc_phase, &bars->abort, a.status);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) {
+                    aborted = true;
                     break;
-                float x[32];
-                ptx::tmem_ld_32x32b_x32(tbase + (uint32_t)(c * 32), x);
-                ptx::tmem_ld_wait();
-                if (cvalid < 32) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (j >= cvalid)
-                            x[j] = -INFINITY;  // columns past V are TMA zero fill, not logits
                 }
-                float cm = x[0];
+                ptx::tc_fence_after();
+                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
+#pragma unroll 1
+                for (int c = 0; c < kBN / 32; ++c) {
+                    const int cvalid = nvalid - c * 32;  // warp-uniform
+                    if (cvalid <= 0)
+                        break;
+                    float x[32];
+                    ptx::tmem_ld_32x32b_x32(tbase + (uint32_t)(c * 32), x);
+                    ptx::tmem_ld_wait();
+                    if (cvalid < 32) {
 #pragma unroll
-                for (int j = 1; j < 32; ++j)
-                    cm = fmaxf(cm, x[j]);
-                if (cm > m) {  // strict: an earlier column keeps the argmax on ties
-                    int j0 = 31;
+                        for (int j = 0; j < 32; ++j)
+                            if (j >= cvalid)
+                                x[j] = -INFINITY;  // columns past V are TMA zero fill, not logits
+                    }
+                    float cm = x[0];
 #pragma unroll
-                    for (int j = 31; j >= 0; --j)
-                        if (x[j] == cm)
-                            j0 = j;
-                    am = v0 + c * 32 + j0;
-                    const float scale = ptx::ex2((m - cm) * kLog2e);
-                    s0 *= scale;
-                    s1 *= scale;
-                    s2 *= scale;
-                    s3 *= scale;
-                    m = cm;
+                    for (int j = 1; j < 32; ++j)
+                        cm = fmaxf(cm, x[j]);
+                    if (cm > m) {  // strict: an earlier column keeps the argmax on ties
+                        int j0 = 31;
+#pragma unroll
+                        for (int j = 31; j >= 0; --j)
+                            if (x[j] == cm)
+                                j0 = j;
+                        am = v0 + c * 32 + j0;
+                        const float scale = ptx::ex2((m - cm) * kLog2e);
+                        s0 *= scale;
+                        s1 *= scale;
+                        s2 *= scale;
+                        s3 *= scale;
+                        m = cm;
+                    }
+                    const float mb2 = m * kLog2e;
+#pragma unroll
+                    for (int j = 0; j < 32; j += 4) {
+                        s0 += ptx::ex2(fmaf(x[j + 0], kLog2e, -mb2));
+                        s1 += ptx::ex2(fmaf(x[j + 1], kLog2e, -mb2));
+                        s2 += ptx::ex2(fmaf(x[j + 2], kLog2e, -mb2));
+                        s3 += ptx::ex2(fmaf(x[j + 3], kLog2e, -mb2));
+                    }
+                    const int tj = tgt - (v0 + c * 32);
+                    if ((unsigned)tj < 32u) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            tl = (j == tj) ? x[j] : tl;
+                    }
                 }
-                const float mb2 = m * kLog2e;
-#pragma unroll
-                for (int j = 0; j < 32; j += 4) {
-                    s0 += ptx::ex2(fmaf(x[j + 0], kLog2e, -mb2));
-                    s1 += ptx::ex2(fmaf(x[j + 1], kLog2e, -mb2));
-                    s2 += ptx::ex2(fmaf(x[j + 2], kLog2e, -mb2));
-                    s3 += ptx::ex2(fmaf(x[j + 3], kLog2e, -mb2));
-                }
-                const int tj = tgt - (v0 + c * 32);
-                if ((unsigned)tj < 32u) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        tl = (j == tj) ? x[j] : tl;
+                // Accumulator fully read: hand it back to the MMA warp.
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    ptx::mbar_arrive(tempty(acc));
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
                 }
             }
-            // Accumulator fully read: hand it back to the MMA warp.
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0)
-                ptx::mbar_arrive(tempty(acc));
-            if (row < a.N)
-                a.part[row * a.n_vt + vt] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tl);
-            if (++acc == 2) {
-                acc = 0;
-                acc_phase ^= 1u;
-            }
+            if (!aborted && row < a.N)
+                a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tl);
         }
         ptx::tc_fence_before();
     }
@@ -317,63 +330,32 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     }
 }
 
-// Fold (m2, s2, i2) into (m, s, i): the larger max wins, the smaller index on equal maxima.
-__device__ __forceinline__ void combine(float &m, float &s, int32_t &i, float m2, float s2, int32_t i2)
-{
-    const float M = fmaxf(m, m2);
-    const float a = (m == -INFINITY) ? 0.f : s * ptx::ex2((m - M) * kLog2e);
-    const float b = (m2 == -INFINITY) ? 0.f : s2 * ptx::ex2((m2 - M) * kLog2e);
-    if (m2 > m || (m2 == m && i2 < i))
-        i = i2;
-    m = M;
-    s = a + b;
-}
-
-// One warp per row: fold the row's per-tile records (fixed lane order, then a
-// butterfly), giving argmax, pmax = 1 / Z and ptarget = exp(l_t - m) / Z.
-__global__ void __launch_bounds__(256) merge_kernel(const float4 *__restrict__ part, int32_t N, int32_t n_vt,
-                                                    int32_t V, const TargetSource ts,
-                                                    const int32_t *__restrict__ status, int32_t *argmax,
-                                                    float *pmax, float *ptarget)
-{
-    const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (row >= N)
-        return;
-    if (status && *status != WINO_OK) {
-        if (lane == 0) {
-            argmax[row] = -1;
-            pmax[row] = __int_as_float(0x7fc00000);
-            ptarget[row] = __int_as_float(0x7fc00000);
-        }
-        return;
-    }
-    const float4 *pr = part + row * n_vt;
-    float m = -INFINITY, s = 0.f;
-    int32_t idx = INT32_MAX;
-    for (int vt = lane; vt < n_vt; vt += 32) {
-        const float4 r = pr[vt];
-        combine(m, s, idx, r.x, r.y, __float_as_int(r.z));
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
-        const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
-        const int32_t i2 = __shfl_xor_sync(0xffffffffu, idx, off);
-        combine(m, s, idx, m2, s2, i2);
-    }
-    if (lane == 0) {
-        const int32_t t = row_target(ts, row, V);
-        argmax[row] = idx;
-        pmax[row] = 1.0f / s;
-        ptarget[row] = (t >= 0) ? ptx::ex2((pr[t / kBN].w - m) * kLog2e) / s : 0.0f;
-    }
-}
-
 }  // namespace
 
-cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, int grid,
-                         cudaStream_t stream)
+// Choose the number of row-block groups: fewest tiles on the busiest CTA,
+// then fewest passes over W (more groups = fewer passes).
+void score_schedule(int32_t n_mb, int32_t n_vt, int max_ctas, int32_t *n_groups, int32_t *G)
+{
+    int64_t best_rounds = -1;
+    int32_t best_groups = 1, best_g = 1;
+    const int32_t top = n_mb < max_ctas ? n_mb : max_ctas;
+    for (int32_t groups = top; groups >= 1; --groups) {
+        int32_t g = max_ctas / groups;
+        g = g < n_vt ? g : n_vt;
+        g = g < kMaxRecordsPerRow ? g : kMaxRecordsPerRow;
+        g = g < 1 ? 1 : g;
+        const int64_t rounds = (int64_t)((n_mb + groups - 1) / groups) * ((n_vt + g - 1) / g);
+        if (best_rounds < 0 || rounds < best_rounds) {
+            best_rounds = rounds;
+            best_groups = groups;
+            best_g = g;
+        }
+    }
+    *n_groups = best_groups;
+    *G = best_g;
+}
+
+cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream)
 {
     static thread_local int configured_device = -1;
     int dev = -1;
@@ -386,16 +368,17 @@ cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const S
             return e;
         configured_device = dev;
     }
-    score_kernel<<<grid, kScoreThreads, kScoreSmemBytes, stream>>>(tmH, tmW, a);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_merge(const float4 *part, int32_t N, int32_t n_vt, int32_t V, const TargetSource &ts,
-                         const int32_t *status, int32_t *argmax, float *pmax, float *ptarget, cudaStream_t stream)
-{
-    const int blocks = (N + 7) / 8;
-    merge_kernel<<<blocks, 256, 0, stream>>>(part, N, n_vt, V, ts, status, argmax, pmax, ptarget);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(a.n_groups * a.G));
+    cfg.blockDim = dim3(kScoreThreads);
+    cfg.dynamicSmemBytes = kScoreSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, score_kernel, tmH, tmW, a);
 }
 
 }  // namespace wino

@@ -23,18 +23,21 @@ constexpr size_t kAlign = 256;
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Workspace layout: [status | partial records [N][n_vt] | argmax[N] | pmax[N] | ptarget[N]].
+// Workspace layout: [status | tickets[ceil(N/2)] | partial records [N][R] | argmax[N] | pmax[N] | ptarget[N]],
+// R = min(ceil(V/kBN), kMaxRecordsPerRow) bounds the records per row of any device.
 struct WsLayout {
-    size_t status, part, argmax, pmax, ptarget, total;
+    size_t status, tickets, part, argmax, pmax, ptarget, total;
 };
 
 WsLayout ws_layout(int64_t N, int64_t V)
 {
     const int64_t n_vt = (V + kBN - 1) / kBN;
+    const int64_t R = n_vt < kMaxRecordsPerRow ? n_vt : kMaxRecordsPerRow;
     WsLayout L{};
     L.status = 0;
-    L.part = kAlign;
-    L.argmax = L.part + round_up((size_t)N * (size_t)n_vt * sizeof(float4), kAlign);
+    L.tickets = kAlign;
+    L.part = L.tickets + round_up((size_t)((N + 1) / 2) * 4, kAlign);
+    L.argmax = L.part + round_up((size_t)N * (size_t)R * sizeof(float4), kAlign);
     L.pmax = L.argmax + round_up((size_t)N * 4, kAlign);
     L.ptarget = L.pmax + round_up((size_t)N * 4, kAlign);
     L.total = L.ptarget + round_up((size_t)N * 4, kAlign);
@@ -184,9 +187,11 @@ int check_params(const wino_params *p)
     return WINO_OK;
 }
 
-// Score N rows into (argmax, pmax, ptarget); steps 1-2 of the WINO step.
-int score_into(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
-               int32_t *argmax, float *pmax, float *ptarget, void *ws, size_t ws_bytes, cudaStream_t stream)
+// Score N rows into (argmax, pmax, ptarget), and with `step` also apply Eq. 4:
+// the score kernel followed by the finish kernel.
+int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
+                     int32_t *argmax, float *pmax, float *ptarget, void *ws, size_t ws_bytes, const wino_params *step,
+                     int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream)
 {
     DeviceInfo info;
     int rc = device_info(&info);
@@ -208,16 +213,34 @@ int score_into(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64
     a.n_mb = (int32_t)((N + kBM - 1) / kBM);
     a.n_vt = (int32_t)((V + kBN - 1) / kBN);
     a.n_kb = (int32_t)((d + kBK - 1) / kBK);
-    a.n_tiles = (int64_t)a.n_mb * a.n_vt;
+    score_schedule(a.n_mb, a.n_vt, info.sm_count, &a.n_groups, &a.G);
     a.ts = ts;
     a.part = reinterpret_cast<float4 *>(w8 + L.part);
     a.status = reinterpret_cast<int32_t *>(w8 + L.status);
-    const int grid = (int)std::min<int64_t>(a.n_tiles, info.sm_count);
+    a.tickets = reinterpret_cast<int32_t *>(w8 + L.tickets);
+    a.n_tickets = step ? step->n_seq : 0;
     prof_record(0, stream);
-    if (launch_score(tmH, tmW, a, grid, stream) != cudaSuccess)
+    if (launch_score(tmH, tmW, a, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
     prof_record(1, stream);
-    if (launch_merge(a.part, a.N, a.n_vt, a.V, ts, a.status, argmax, pmax, ptarget, stream) != cudaSuccess)
+    FinishArgs f{};
+    f.part = a.part;
+    f.G = a.G;
+    f.N = a.N;
+    f.V = a.V;
+    f.ts = ts;
+    f.status = a.status;
+    f.argmax = argmax;
+    f.pmax = pmax;
+    f.ptarget = ptarget;
+    if (step) {
+        f.tokens = tokens;
+        f.p = *step;
+        f.counts = counts;
+        f.flags = flags;
+        f.tickets = a.tickets;
+    }
+    if (launch_finish(f, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
     return WINO_OK;
 }
@@ -267,7 +290,8 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
         return WINO_ERR_SHAPE;
     TargetSource ts{};
     ts.target = target;
-    return score_into(H, W, N, d, V, ts, argmax, pmax, ptarget, ws, ws_bytes, static_cast<cudaStream_t>(stream));
+    return score_and_finish(H, W, N, d, V, ts, argmax, pmax, ptarget, ws, ws_bytes, nullptr, nullptr, nullptr,
+                            nullptr, static_cast<cudaStream_t>(stream));
 }
 
 int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
@@ -281,8 +305,8 @@ int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax,
     DeviceInfo info;
     if ((rc = device_info(&info)) != WINO_OK)
         return rc;
-    if (launch_draft_verify(tokens, argmax, pmax, ptarget, *p, counts, flags, nullptr,
-                            static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    if (launch_draft_verify(tokens, argmax, pmax, ptarget, *p, counts, flags, static_cast<cudaStream_t>(stream)) !=
+        cudaSuccess)
         return WINO_ERR_CUDA;
     return WINO_OK;
 }
@@ -313,13 +337,8 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     ts.blk_start = p->blk_start;
     ts.blk_len = p->blk_len;
     ts.mask_id = p->mask_id;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if ((rc = score_into(H, W, N, d, V, ts, am, pm, pt, ws, ws_bytes, s)) != WINO_OK)
-        return rc;
-    if (launch_draft_verify(tokens, am, pm, pt, *p, counts, flags, reinterpret_cast<const int32_t *>(w8 + L.status),
-                            s) != cudaSuccess)
-        return WINO_ERR_CUDA;
-    return WINO_OK;
+    return score_and_finish(H, W, N, d, V, ts, am, pm, pt, ws, ws_bytes, p, tokens, counts, flags,
+                            static_cast<cudaStream_t>(stream));
 }
 
 int wino_profile_begin(int max_launches)

@@ -1,7 +1,10 @@
 """Semi-autoregressive WINO decode loop over the C ABI (Sec. 3 and Sec. 4.2.3).
 
 Blocks are decoded left to right; inside a block ``wino_step`` is repeated
-until no position of the block is MASK in any sequence of the batch.  The
+until no position of the block is MASK in any sequence of the batch.  A
+sequence whose block is complete is frozen (WINO_OPT_FREEZE_FINISHED): its
+own loop has ended, so it is not re-verified while the rest of the batch
+finishes the block.  The
 only device-to-host traffic per step is the [n_seq, 3] counts array, read to
 decide whether the block is finished.  The hidden states of each step come
 from a caller-supplied function (the transformer forward with the
@@ -55,7 +58,7 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     k = 0
     for b in range(n_blocks):
         b0 = prompt_len + b * blk_len
-        p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps)
+        p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True)
         bs = BlockStats(block=b, blk_start=b0)
         while True:
             if bs.steps >= max_steps:

@@ -335,7 +335,22 @@ def pin_loop_terminates(O):
     assert not np.any(tokens[:, w.prompt_len:] == w.mask_id)
 
 
-EQ4_PINS = [pin_eq4_hand_cases, pin_only_draft_never_remasks, pin_greedy_reduction,
+def pin_freeze_finished(O):
+    """A sequence whose block has no MASK has finished its loop (Sec. 4.2.3): with the
+    freeze option it is not stepped; without it Eq. 4 still verifies it."""
+    M = 9
+    tokens = np.array([[1, 2, 3, 4], [1, M, 3, 4]], np.int32)
+    am = _rows(2, 3, [[5, 5, 5], [6, 6, 6]], [[0] * 3, [0] * 3])
+    pm = _rows(2, 3, [[0.9] * 3, [0.9] * 3], [[0.0] * 3, [0.0] * 3])
+    pt = _rows(2, 3, [[0.0] * 3, [0.0] * 3], [[0.1, 0.1, 0.95], [0.1, 0.1, 0.1]])
+    tok, cnt, fl = O.draft_verify(tokens, 1, 3, M, 0.5, 0.9, am, pm, pt, freeze_finished=True)
+    assert tok.tolist() == [[1, 2, 3, 4], [1, 6, M, M]], tok
+    assert cnt.tolist() == [[0, 0, 0], [1, 2, 2]] and fl.tolist() == [[0, 0, 0], [1, 3, 3]], (cnt, fl)
+    tok, cnt, fl = O.draft_verify(tokens, 1, 3, M, 0.5, 0.9, am, pm, pt, freeze_finished=False)
+    assert tok.tolist() == [[1, M, M, 4], [1, 6, M, M]] and cnt.tolist() == [[0, 2, 2], [1, 2, 2]], (tok, cnt)
+
+
+EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_only_draft_never_remasks, pin_greedy_reduction,
             pin_eq4_exhaustive_properties, pin_loop_terminates]
 
 ALL_PINS = SCORING_PINS + EQ4_PINS

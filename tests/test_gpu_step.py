@@ -27,20 +27,23 @@ CASES = [(1, 1, 3, 1), (1, 32, 40, 4), (5, 31, 70, 2), (17, 33, 100, 50), (3, 12
 
 @pytest.mark.parametrize("n_seq,L,S,b0", CASES, ids=[f"B{c[0]}_L{c[1]}" for c in CASES])
 @pytest.mark.parametrize("taus", [(0.5, 0.75), (0.7, 0.9), (1.0, 0.0), (0.0, 1.0)], ids=str)
-def test_draft_verify_bit_exact(n_seq, L, S, b0, taus):
+@pytest.mark.parametrize("freeze", [False, True], ids=["eq4", "freeze"])
+def test_draft_verify_bit_exact(n_seq, L, S, b0, taus, freeze):
     """Given the same fp32 statistics, the kernel's Eq. 4 equals the oracle's bit for bit."""
     import paper_2605_16941_gb300 as wino
     from gpu_helpers import dev, f32, host
     M = 997
     rng = np.random.default_rng(n_seq * 1000 + L)
     tokens, am, pm, pt = _random_case(rng, n_seq, L, S, b0, M)
+    if freeze and n_seq > 1:
+        tokens[0, b0:b0 + L] = rng.integers(0, M, size=L)  # a finished block
     t1, t2 = taus
     ref_tok, ref_cnt, ref_fl = oracle.draft_verify(tokens, b0, L, M, f32(t1), f32(t2), am, pm.astype(np.float64),
-                                                   pt.astype(np.float64))
+                                                   pt.astype(np.float64), freeze_finished=freeze)
     tok_d = dev(tokens)
     counts = torch.full((n_seq, 3), -9, dtype=torch.int32, device="cuda")
     flags = torch.full((n_seq, L), -9, dtype=torch.int8, device="cuda")
-    p = wino.make_params(t1, t2, M, n_seq, S, b0, L)
+    p = wino.make_params(t1, t2, M, n_seq, S, b0, L, freeze_finished=freeze)
     wino.wino_draft_verify(tok_d, dev(am), dev(pm), dev(pt), p, counts, flags)
     torch.cuda.synchronize()
     assert np.array_equal(host(tok_d), ref_tok)
@@ -185,7 +188,8 @@ def test_decode_loop_tiny_lockstep():
     reports = []
 
     def on_step(k, b0, counts, flags):
-        o = oracle.step(record["H"], W, record["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2)
+        o = oracle.step(record["H"], W, record["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2,
+                        freeze_finished=True)
         reports.append(compare_step(record["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1,
                                     w.tau2))
 
@@ -237,7 +241,7 @@ def test_decode_loop_b16():
             t = oracle.row_targets(pre, b0, L, w.mask_id)
             g = gpu_score(rec["Hd"], Wd, t)
             ref = oracle.draft_verify(pre, b0, L, w.mask_id, f32(w.tau1), f32(w.tau2), g.argmax,
-                                      g.pmax.astype(np.float64), g.ptarget.astype(np.float64))
+                                      g.pmax.astype(np.float64), g.ptarget.astype(np.float64), freeze_finished=True)
             assert np.array_equal(post, ref[0]) and np.array_equal(counts, ref[1])
             rows = np.random.default_rng(k).choice(w.N, 8, replace=False)
             compare_rows(oracle.score_rows(rec["H"][rows], W, t[rows]), g, rows)

@@ -40,6 +40,8 @@ MUTANTS = [
      "target[(s * 2 + 0) * blk_len + l] = (y == mask_id) ? -1 : y;"),
     ("remask_not_counted", "++remasked;", ""),
     ("left_counts_old_state", "left += (y[l] == mask_id);", "left += (prev[l] == mask_id);"),
+    ("freeze_ignored", "if (freeze_finished && n_mask == 0) {", "if (0) {"),
+    ("freeze_always", "if (freeze_finished && n_mask == 0) {", "if (n_mask == 0) {"),
 ]
 
 
