@@ -15,7 +15,7 @@
 // results before touching them.
 //
 // draft_verify_kernel: Eq. 4 alone from caller-supplied statistics
-// (wino_draft_verify).
+// (wino_draft_verify), one CTA per sequence.
 //
 // Eq. 4, per sequence, reading the state before the step y^(k-1):
 //   draft  (Eq. 2): y_l == MASK and pmax(block row l) > tau1      -> argmax(block row l)
@@ -24,7 +24,7 @@
 // the masked position with the largest pmax (smallest position on ties) is
 // drafted: the greedy rule of Eq. 1, which keeps at least one token coming per
 // step.  The rules touch disjoint positions (MASK vs not MASK), so the update
-// is applied in place in one pass after a warp-wide reduction.  With
+// is applied in place in one pass after a CTA-wide reduction.  With
 // WINO_OPT_FREEZE_FINISHED a sequence whose block already has no MASK is left
 // as it is (its own loop, Sec. 4.2.3, has ended).
 #include "internal.h"
@@ -34,8 +34,7 @@ namespace wino {
 namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int kFinishRows = 8;  // rows (warps) per finish CTA
-constexpr int kDVWarps = 4;     // sequences (warps) per draft_verify CTA
+constexpr int kFinishRows = 8;  // rows (warps) per finish CTA; also the CTA size of the Eq. 4 kernels
 
 // Fold (m2, s2, i2) into (m, s, i): the larger max wins, the smaller index on equal maxima.
 __device__ __forceinline__ void combine(float &m, float &s, int32_t &i, float m2, float s2, int32_t i2)
@@ -49,14 +48,24 @@ __device__ __forceinline__ void combine(float &m, float &s, int32_t &i, float m2
     s = a + b;
 }
 
-// Eq. 4 on sequence s by one warp.  Statistics are read through L2 (other CTAs may have written them).
-__device__ void eq4_sequence(int s, int lane, int32_t *tokens, const int32_t *argmax, const float *pmax,
-                             const float *ptarget, const wino_params &p, int32_t *counts, int8_t *flags,
-                             int32_t status)
+// Block-wide reduction scratch for eq4_block.
+struct Eq4Smem {
+    int32_t i0[kFinishRows], i1[kFinishRows], i2[kFinishRows];
+    float f0[kFinishRows];
+};
+
+// Eq. 4 on sequence s by the whole CTA (kFinishRows warps; thread t owns positions t, t + 256, ...).
+// Every load is issued before any decision so the update costs about one memory round trip.
+// Statistics are read through L2: other CTAs of the same launch may have written them.
+__device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
+                          const wino_params &p, int32_t *counts, int8_t *flags, int32_t status, Eq4Smem &sm)
 {
+    constexpr int kT = kFinishRows * 32;
+    constexpr int kPer = kMaxBlkLen / kT;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (status != WINO_OK) {  // the scores of this step are invalid: leave the state alone
-        if (lane < 3)
-            counts[s * 3 + lane] = status;
+        if (tid < 3)
+            counts[s * 3 + tid] = status;
         return;
     }
     const int L = p.blk_len;
@@ -65,17 +74,30 @@ __device__ void eq4_sequence(int s, int lane, int32_t *tokens, const int32_t *ar
     const int64_t rb = (int64_t)(2 * s) * L;      // kind-0 rows: the block Y_cur
     const int64_t rs = (int64_t)(2 * s + 1) * L;  // kind-1 rows: the shadow block Y_shad
 
+    int32_t yv[kPer], av[kPer];
+    float pm[kPer], pt[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int l = tid + i * kT;
+        if (l < L) {
+            yv[i] = y[l];
+            av[i] = __ldcg(argmax + rb + l);
+            pm[i] = __ldcg(pmax + rb + l);
+            pt[i] = __ldcg(ptarget + rs + l);
+        }
+    }
     // Pass 1: how many masked positions clear tau1, and the most confident masked position.
     int n_clear = 0, n_mask = 0;
     float best = -INFINITY;
     int best_l = INT32_MAX;
-    for (int l = lane; l < L; l += 32) {
-        if (y[l] == mask) {
-            const float pm = __ldcg(pmax + rb + l);
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int l = tid + i * kT;
+        if (l < L && yv[i] == mask) {
             ++n_mask;
-            n_clear += (pm > p.tau1);
-            if (pm > best || (pm == best && l < best_l)) {
-                best = pm;
+            n_clear += (pm[i] > p.tau1);
+            if (pm[i] > best) {  // l grows with i: the first maximum keeps the smallest position
+                best = pm[i];
                 best_l = l;
             }
         }
@@ -91,28 +113,52 @@ __device__ void eq4_sequence(int s, int lane, int32_t *tokens, const int32_t *ar
             best_l = l2;
         }
     }
+    if (lane == 0) {
+        sm.i0[warp] = n_clear;
+        sm.i1[warp] = n_mask;
+        sm.i2[warp] = best_l;
+        sm.f0[warp] = best;
+    }
+    __syncthreads();
+    n_clear = n_mask = 0;
+    best = -INFINITY;
+    best_l = INT32_MAX;
+#pragma unroll
+    for (int w = 0; w < kFinishRows; ++w) {
+        n_clear += sm.i0[w];
+        n_mask += sm.i1[w];
+        if (sm.f0[w] > best || (sm.f0[w] == best && sm.i2[w] < best_l)) {
+            best = sm.f0[w];
+            best_l = sm.i2[w];
+        }
+    }
+    __syncthreads();  // the scratch is reused below
     if (n_mask == 0 && (p.options & WINO_OPT_FREEZE_FINISHED)) {  // finished block: its loop has stopped
         if (flags)
-            for (int l = lane; l < L; l += 32)
+            for (int l = tid; l < L; l += kT)
                 flags[(int64_t)s * L + l] = 0;
-        if (lane < 3)
-            counts[s * 3 + lane] = 0;
+        if (tid < 3)
+            counts[s * 3 + tid] = 0;
         return;
     }
     const int fallback = (n_clear == 0 && n_mask > 0) ? best_l : -1;
 
     // Pass 2: apply Eq. 4 simultaneously.
     int drafted = 0, remasked = 0, left = 0;
-    for (int l = lane; l < L; l += 32) {
-        const int32_t prev = y[l];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int l = tid + i * kT;
+        if (l >= L)
+            break;
+        const int32_t prev = yv[i];
         int32_t next = prev;
         int8_t code = 0;
         if (prev == mask) {
-            if (__ldcg(pmax + rb + l) > p.tau1 || l == fallback) {
-                next = __ldcg(argmax + rb + l);
+            if (pm[i] > p.tau1 || l == fallback) {
+                next = av[i];
                 code = (next == mask) ? 4 : (l == fallback ? 2 : 1);
             }
-        } else if (__ldcg(ptarget + rs + l) < p.tau2) {
+        } else if (pt[i] < p.tau2) {
             next = mask;
             code = 3;
         }
@@ -128,10 +174,20 @@ __device__ void eq4_sequence(int s, int lane, int32_t *tokens, const int32_t *ar
     remasked = __reduce_add_sync(0xffffffffu, remasked);
     left = __reduce_add_sync(0xffffffffu, left);
     if (lane == 0) {
-        counts[s * 3 + 0] = drafted;
-        counts[s * 3 + 1] = remasked;
-        counts[s * 3 + 2] = left;
+        sm.i0[warp] = drafted;
+        sm.i1[warp] = remasked;
+        sm.i2[warp] = left;
     }
+    __syncthreads();
+    if (tid < 3) {
+        const int32_t *src = tid == 0 ? sm.i0 : (tid == 1 ? sm.i1 : sm.i2);
+        int32_t v = 0;
+#pragma unroll
+        for (int w = 0; w < kFinishRows; ++w)
+            v += src[w];
+        counts[s * 3 + tid] = v;
+    }
+    __syncthreads();  // the scratch may be reused for the next sequence
 }
 
 __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishArgs a)
@@ -140,6 +196,7 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
     ptx::grid_dep_launch_dependents();
     __shared__ int32_t s_done[kFinishRows];
     __shared__ int32_t s_ndone;
+    __shared__ Eq4Smem sm;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t row0 = (int64_t)blockIdx.x * kFinishRows;
     const int64_t row = row0 + warp;
@@ -154,12 +211,26 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
             }
         } else {
             const float4 *pr = a.part + row * a.G;
+            // every record of the row (G <= 8 * 32) and the target's record are loaded at once
+            constexpr int kRec = kMaxRecordsPerRow / 32;
+            float4 r[kRec];
+#pragma unroll
+            for (int i = 0; i < kRec; ++i) {
+                const int j = lane + 32 * i;
+                r[i] = (j < a.G) ? __ldcg(pr + j) : make_float4(-INFINITY, 0.f, __int_as_float(INT32_MAX), 0.f);
+            }
+            int32_t t = -1;
+            float tl = 0.f;
+            if (lane == 0) {
+                t = row_target(a.ts, row, a.V);
+                if (t >= 0)
+                    tl = __ldcg(pr + (t / kBN) % a.G).w;
+            }
             float m = -INFINITY, s = 0.f;
             int32_t idx = INT32_MAX;
-            for (int j = lane; j < a.G; j += 32) {
-                const float4 r = __ldcg(pr + j);
-                combine(m, s, idx, r.x, r.y, __float_as_int(r.z));
-            }
+#pragma unroll
+            for (int i = 0; i < kRec; ++i)
+                combine(m, s, idx, r[i].x, r[i].y, __float_as_int(r[i].z));
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) {
                 const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
@@ -168,10 +239,9 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
                 combine(m, s, idx, m2, s2, i2);
             }
             if (lane == 0) {
-                const int32_t t = row_target(a.ts, row, a.V);
                 a.argmax[row] = idx;
                 a.pmax[row] = 1.0f / s;
-                a.ptarget[row] = (t >= 0) ? ptx::ex2((__ldcg(pr + (t / kBN) % a.G).w - m) * kLog2e) / s : 0.0f;
+                a.ptarget[row] = (t >= 0) ? ptx::ex2((tl - m) * kLog2e) / s : 0.0f;
                 __threadfence();  // publish this row before the CTA signals its ticket
             }
         }
@@ -197,17 +267,18 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
         __threadfence();
     }
     __syncthreads();
-    for (int i = warp; i < s_ndone; i += kFinishRows)
-        eq4_sequence(s_done[i], lane, a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status);
+    const int nd = s_ndone;
+    for (int i = 0; i < nd; ++i)
+        eq4_block(s_done[i], a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status, sm);
 }
 
-__global__ void __launch_bounds__(kDVWarps * 32)
+// Eq. 4 alone, one CTA per sequence.
+__global__ void __launch_bounds__(kFinishRows * 32)
     draft_verify_kernel(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                         const wino_params p, int32_t *counts, int8_t *flags)
 {
-    const int s = blockIdx.x * kDVWarps + (threadIdx.x >> 5);
-    if (s < p.n_seq)
-        eq4_sequence(s, threadIdx.x & 31, tokens, argmax, pmax, ptarget, p, counts, flags, WINO_OK);
+    __shared__ Eq4Smem sm;
+    eq4_block(blockIdx.x, tokens, argmax, pmax, ptarget, p, counts, flags, WINO_OK, sm);
 }
 
 }  // namespace
@@ -230,8 +301,7 @@ cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream)
 cudaError_t launch_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                                 const wino_params &p, int32_t *counts, int8_t *flags, cudaStream_t stream)
 {
-    const int blocks = (p.n_seq + kDVWarps - 1) / kDVWarps;
-    draft_verify_kernel<<<blocks, kDVWarps * 32, 0, stream>>>(tokens, argmax, pmax, ptarget, p, counts, flags);
+    draft_verify_kernel<<<p.n_seq, kFinishRows * 32, 0, stream>>>(tokens, argmax, pmax, ptarget, p, counts, flags);
     return cudaGetLastError();
 }
 
