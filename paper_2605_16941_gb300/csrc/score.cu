@@ -34,7 +34,6 @@ namespace {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait
 constexpr uint64_t kDrainLimitNs = 200000000ull;   // 0.2 s for draining after an abort
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int64_t kPrefetchAhead = 8;  // W slices (256 x 64 bf16 = 32 KB each) pulled into L2 ahead of the ring
 
 struct alignas(8) Barriers {
     uint64_t full[kStages];
@@ -145,21 +144,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             issued_parity[s] = -1;
         bool aborted = false;
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-            // W slices of this row block in issue order: i -> (vocab tile col + (i / n_kb) * G, K block i % n_kb).
-            // Slice i + kPrefetchAhead is pulled into L2 when slice i is issued, so the ring's loads find W in
-            // L2 instead of waiting on HBM.
-            const int64_t n_slices = (int64_t)((a.n_vt - col + a.G - 1) / a.G) * a.n_kb;
-            auto prefetch_w = [&](int64_t i) {
-                if (lane == 0 && i < n_slices)
-                    ptx::tma_prefetch_l2_2d(&tmW, (int32_t)(i % a.n_kb) * kBK,
-                                            (int32_t)(col + (i / a.n_kb) * a.G) * kBN);
-            };
-            for (int64_t i = 0; i < kPrefetchAhead; ++i)
-                prefetch_w(i);
-            int64_t slice = 0;
             for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
-                for (int kb = 0; kb < a.n_kb; ++kb, ++slice) {
-                    prefetch_w(slice + kPrefetchAhead);
+                for (int kb = 0; kb < a.n_kb; ++kb) {
                     int ok = 1;
                     if (lane == 0)
                         ok = wait_bounded(empty(stage), phase ^ 1u, &bars->abort, a.status);
