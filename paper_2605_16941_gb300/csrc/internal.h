@@ -10,19 +10,23 @@
 
 namespace wino {
 
-// Scoring tile: 128 rows of H (one TMEM lane each) x 256 vocabulary columns
-// (the UMMA N extent and one 256-column TMEM accumulator), K staged 64 bf16
-// (one 128-byte swizzle row) at a time through a 4-deep shared-memory ring.
-constexpr int kBM = 128;
-constexpr int kBN = 256;
+// Scoring tile: a CTA pair (2-SM tcgen05 MMA, cta_group::2) computes 256 rows
+// of H x 256 vocabulary columns.  Each CTA stages its own 128 rows of H and 128
+// of the 256 W rows per 64-wide K slice (128-byte swizzle rows) through a
+// 6-deep shared-memory ring, and holds its 128 rows x 256 columns of the fp32
+// accumulator in TMEM (one TMEM lane per row).
+constexpr int kPairM = 256;  // rows per pair tile (UMMA M)
+constexpr int kBM = 128;     // rows per CTA
+constexpr int kBN = 256;     // vocabulary columns per tile (UMMA N)
+constexpr int kHalfN = 128;  // W rows staged by each CTA of the pair
 constexpr int kBK = 64;
-constexpr int kStages = 4;
-constexpr int kScoreThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
-constexpr uint32_t kStageBytesA = kBM * kBK * 2;  // 16 KB
-constexpr uint32_t kStageBytesB = kBN * kBK * 2;  // 32 KB
+constexpr int kStages = 6;
+constexpr int kScoreThreads = 192;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 epilogue
+constexpr uint32_t kStageBytesA = kBM * kBK * 2;     // 16 KB
+constexpr uint32_t kStageBytesB = kHalfN * kBK * 2;  // 16 KB
 constexpr uint32_t kRingBytes = kStages * (kStageBytesA + kStageBytesB);
 constexpr uint32_t kScoreSmemBytes = kRingBytes + 1024 /* alignment slack */ + 256 /* barriers */;
-constexpr uint32_t kTmemCols = 2 * kBN;  // double-buffered fp32 accumulator
+constexpr uint32_t kTmemCols = kBN;  // one 256-column fp32 accumulator
 
 constexpr int kMaxBlkLen = 1024;
 
@@ -51,20 +55,20 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
     return (t >= 0 && t < V) ? t : -1;
 }
 
-// Work split of the score kernel.  The row blocks are spread over n_groups
-// groups of G CTAs; CTA c serves row blocks c % n_groups (+ n_groups, ...) and,
-// within each, vocabulary tiles c / n_groups (+ G, ...).  The G CTAs of a group
-// walk the vocabulary side by side, so all groups read the same W tiles at the
-// same time (W streams from HBM about once), and each CTA keeps its running
-// softmax state per row across its tiles and writes ONE partial record per
-// (row, CTA of the group): G records per row.
+// Work split of the score kernel.  The 256-row blocks are spread over n_groups
+// groups of G CTA pairs; pair c serves row blocks c % n_groups (+ n_groups, ...)
+// and, within each, vocabulary tiles c / n_groups (+ G, ...).  The G pairs of a
+// group walk the vocabulary side by side, so all groups read the same W tiles
+// at the same time (W streams from HBM about once), and each CTA keeps its
+// running softmax state per row across its tiles and writes ONE partial record
+// per (row, pair of the group): G records per row.
 constexpr int kMaxRecordsPerRow = 256;
 
 // Partial record: running max logit m, sum of exp(l - m), argmax (int bits),
 // logit of the row's target if the target lies in one of the CTA's tiles (else 0).
 struct ScoreArgs {
     int32_t N, d, V;
-    int32_t n_mb, n_vt, n_kb;
+    int32_t n_mb, n_vt, n_kb;  // n_mb: 256-row blocks
     int32_t n_groups, G;
     TargetSource ts;
     float4 *part;       // [N][G]
@@ -89,7 +93,10 @@ struct FinishArgs {
     int32_t *tickets;  // [n_seq], zero on entry
 };
 
-void score_schedule(int32_t n_mb, int32_t n_vt, int max_ctas, int32_t *n_groups, int32_t *G);
+void score_schedule(int32_t n_mb, int32_t n_vt, int max_units, int32_t *n_groups, int32_t *G);
+
+// CTA pairs of the score kernel that can be resident at once on the current device (<= 0 on error).
+int score_max_pairs();
 
 cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream);
 

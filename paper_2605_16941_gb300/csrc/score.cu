@@ -3,28 +3,30 @@
 // For every scored row h_n the method needs three numbers of the model's
 // distribution p(. | Y~) = softmax_v(<h_n, w_v>) over the whole vocabulary
 // (Eq. 2 and Eq. 3 of the WINO paper): argmax_v p, max_v p and p(target).
-// The logits never leave the chip: each CTA computes 128 x 256 logit tiles
-// on the tensor cores (tcgen05.mma, bf16 x bf16 -> fp32 in TMEM), and four
-// epilogue warps fold each tile straight out of TMEM into a running
+// The logits never leave the chip: each CTA pair computes 256 x 256 logit
+// tiles with 2-SM tensor-core MMAs (tcgen05.mma.cta_group::2, bf16 x bf16 ->
+// fp32 in TMEM, M = 256 split 128/128 over the two SMs, N = 256), and four
+// epilogue warps per CTA fold each tile straight out of TMEM into a running
 // per-row state (max, sum of exp, argmax, target logit) that lives in
-// registers across all of the CTA's vocabulary tiles of that row block.  One
-// partial record per (row, CTA) goes to the workspace; finish.cu merges them.
+// registers across all of the pair's vocabulary tiles of that row block.  One
+// partial record per (row, pair) goes to the workspace; finish.cu merges them.
 //
-// Kernel structure (persistent, one CTA per SM, 192 threads):
-//   warp 0  TMA producer: streams 64-wide K slices of H (128 rows) and W
-//           (256 vocabulary rows) into a 4-stage shared-memory ring;
-//   warp 1  MMA issuer: allocates 512 TMEM columns (two 256-column fp32
-//           accumulators), issues 4 x (M128 N256 K16) MMAs per stage and
-//           commits stage-release / accumulator-ready barriers;
-//   warps 2-5 epilogue: one thread per row (TMEM lane), online softmax over
-//           each tile's 256 columns while the MMA warp fills the other
-//           accumulator.
-// Work split: see ScoreArgs in internal.h (row-block groups walking the
-// vocabulary side by side).
+// Kernel structure (persistent, clusters of 2 CTAs = one SM pair, 192 threads each):
+//   warp 0  TMA producer (both CTAs): streams 64-wide K slices of its 128 rows
+//           of H and of its 128 of the tile's 256 W rows into a 6-stage ring;
+//           both CTAs' copies complete on the LEADER's stage barrier;
+//   warp 1  TMEM allocation (both CTAs) and, in the leader only, the MMA
+//           issuer: 4 x (M256 N256 K16) per stage, committing stage release
+//           and accumulator-ready to both CTAs (multicast);
+//   warps 2-5 epilogue (both CTAs): one thread per row (TMEM lane); online
+//           softmax over the tile's 256 columns, then release the
+//           accumulator to the leader's MMA warp (8 arrivals per tile).
+// Work split: see ScoreArgs in internal.h.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA raises an
 // abort flag, records WINO_ERR_DEVICE_TIMEOUT in the status word, drains its
-// in-flight copies and MMAs (again bounded) and frees its TMEM.
+// in-flight copies and MMAs (again bounded); both CTAs then meet at the
+// closing cluster barrier before TMEM is released.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -34,27 +36,30 @@ namespace {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait
 constexpr uint64_t kDrainLimitNs = 200000000ull;   // 0.2 s for draining after an abort
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr uint16_t kBothCtas = 0x3;
 
 struct alignas(8) Barriers {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
-    uint64_t tmem_full[2];
-    uint64_t tmem_empty[2];
-    uint64_t mma_done;
+    uint64_t full[kStages];   // leader: both CTAs' copies of a stage landed
+    uint64_t empty[kStages];  // both: the stage's MMAs are done (multicast commit)
+    uint64_t tmem_full;       // both: the accumulator holds a finished tile (multicast commit)
+    uint64_t tmem_empty;      // leader: all 8 epilogue warps of the pair have read the accumulator
+    uint64_t mma_done;        // leader: every MMA issued has completed
     uint32_t tmem_base;
     int32_t abort;
 };
 static_assert(sizeof(Barriers) <= 256, "barrier block must fit its reserve");
 
 // Wait for phase `parity` of `bar`; false once the wait limit passed or another
-// role of this CTA aborted.
+// role of this CTA aborted.  kCluster: acquire at cluster scope (barrier arrived on by the peer CTA).
+template <bool kCluster = false>
 __device__ bool wait_bounded(uint32_t bar, uint32_t parity, int32_t *abort_flag, int32_t *status)
 {
-    if (ptx::mbar_try_wait(bar, parity))
+    auto try_wait = [&] { return kCluster ? ptx::mbar_try_wait_cluster(bar, parity) : ptx::mbar_try_wait(bar, parity); };
+    if (try_wait())
         return true;
     const uint64_t t0 = ptx::globaltimer_ns();
     for (uint32_t it = 1;; ++it) {
-        if (ptx::mbar_try_wait(bar, parity))
+        if (try_wait())
             return true;
         if ((it & 15u) == 0) {
             if (*reinterpret_cast<volatile int32_t *>(abort_flag))
@@ -87,13 +92,17 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const uint32_t ring = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-B alignment
     Barriers *bars = reinterpret_cast<Barriers *>(smem_raw + (ring - raw) + kRingBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = ptx::cluster_ctarank();  // 0: leader (issues the MMAs), 1: peer
+    const bool leader = rank == 0;
+    const int pair = blockIdx.x >> 1;
 
     auto sA = [&](int s) { return ring + (uint32_t)s * (kStageBytesA + kStageBytesB); };
     auto sB = [&](int s) { return sA(s) + kStageBytesA; };
     auto full = [&](int s) { return ptx::smem_u32(&bars->full[s]); };
     auto empty = [&](int s) { return ptx::smem_u32(&bars->empty[s]); };
-    auto tfull = [&](int s) { return ptx::smem_u32(&bars->tmem_full[s]); };
-    auto tempty = [&](int s) { return ptx::smem_u32(&bars->tmem_empty[s]); };
+    const uint32_t tfull = ptx::smem_u32(&bars->tmem_full);
+    const uint32_t tempty = ptx::smem_u32(&bars->tmem_empty);
+    const uint32_t mma_done = ptx::smem_u32(&bars->mma_done);
 
     // Set-up that touches no global memory overlaps the previous kernel (programmatic launch).
     if (threadIdx.x == 0) {
@@ -101,11 +110,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             ptx::mbar_init(full(s), 1);
             ptx::mbar_init(empty(s), 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            ptx::mbar_init(tfull(s), 1);
-            ptx::mbar_init(tempty(s), 4);  // one arrival per epilogue warp
-        }
-        ptx::mbar_init(ptx::smem_u32(&bars->mma_done), 1);
+        ptx::mbar_init(tfull, 1);
+        ptx::mbar_init(tempty, 8);  // 4 epilogue warps in each CTA of the pair
+        ptx::mbar_init(mma_done, 1);
         bars->abort = 0;
         ptx::fence_barrier_init();
     }
@@ -114,27 +121,35 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         ptx::prefetch_tensormap(&tmW);
     }
     if (warp == 1) {
-        ptx::tmem_alloc(ptx::smem_u32(&bars->tmem_base), kTmemCols);
-        ptx::tmem_relinquish();
+        // Both CTAs of the pair take part in the pair allocation.  256 columns: even if each CTA's
+        // request were served separately in both SMs, 2 x 256 fits the 512 columns of an SM, and the
+        // address check below then refuses to run.
+        ptx::tmem_alloc_pair(ptx::smem_u32(&bars->tmem_base), kTmemCols);
+        ptx::tmem_relinquish_pair();
     }
     ptx::tc_fence_before();
-    __syncthreads();
+    ptx::cluster_sync();  // barriers and TMEM address of both CTAs are now visible to both
     ptx::tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
+    const uint32_t peer_tmem = ptx::ld_shared_cluster_u32(ptx::mapa(ptx::smem_u32(&bars->tmem_base), rank ^ 1u));
+    const bool tmem_ok = (peer_tmem == tmem);
 
     // From here on global memory is read and written: wait for the grid before us.
     ptx::grid_dep_wait();
     ptx::grid_dep_launch_dependents();
     if (blockIdx.x == 0 && threadIdx.x == 0)
-        *a.status = WINO_OK;  // a timeout, if any, is raised no earlier than kWaitLimitNs later
+        *a.status = tmem_ok ? WINO_OK : WINO_ERR_UNSUPPORTED;
     for (int i = blockIdx.x * kScoreThreads + threadIdx.x; i < a.n_tickets; i += gridDim.x * kScoreThreads)
         a.tickets[i] = 0;
 
-    const int grp = blockIdx.x % a.n_groups;  // row blocks grp, grp + n_groups, ...
-    const int col = blockIdx.x / a.n_groups;  // vocabulary tiles col, col + G, ...
+    const int grp = pair % a.n_groups;  // 256-row blocks grp, grp + n_groups, ...
+    const int col = pair / a.n_groups;  // vocabulary tiles col, col + G, ...
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
+    if (!tmem_ok) {
+        if (threadIdx.x == 0)
+            atomicExch(a.status, (int32_t)WINO_ERR_UNSUPPORTED);
+    } else if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer (both CTAs)
         const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every vocabulary tile
         const uint64_t pol_w = ptx::policy_evict_normal();  // W is shared by the row-block groups
         int stage = 0;
@@ -155,9 +170,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         break;
                     }
                     if (lane == 0) {
-                        ptx::mbar_arrive_expect_tx(full(stage), kStageBytesA + kStageBytesB);
-                        ptx::tma_load_2d(sA(stage), &tmH, full(stage), kb * kBK, mb * kBM, pol_h);
-                        ptx::tma_load_2d(sB(stage), &tmW, full(stage), kb * kBK, vt * kBN, pol_w);
+                        const uint32_t bar = ptx::mapa(full(stage), 0);  // the leader's stage barrier
+                        if (leader)
+                            ptx::mbar_arrive_expect_tx(full(stage), 2 * (kStageBytesA + kStageBytesB));
+                        ptx::tma_load_2d_pair(sA(stage), &tmH, bar, kb * kBK, mb * kPairM + (int)rank * kBM, pol_h);
+                        ptx::tma_load_2d_pair(sB(stage), &tmW, bar, kb * kBK, vt * kBN + (int)rank * kHalfN,
+                                              pol_w);
                     }
                     __syncwarp();
                     issued_parity[stage] = (int32_t)phase;
@@ -168,82 +186,79 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 }
             }
         }
-        if (aborted && lane == 0) {
-            // Let every copy already issued land before the CTA (and its shared memory) goes away.
+        if (aborted && leader && lane == 0) {
+            // Let every copy already issued (by either CTA) land before the pair's shared memory goes away.
             for (int s = 0; s < kStages; ++s)
                 if (issued_parity[s] >= 0)
                     wait_drain(full(s), (uint32_t)issued_parity[s]);
         }
         __syncwarp();
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        constexpr uint32_t idesc = ptx::idesc_bf16_f32(kBM, kBN);
-        int stage = 0;
-        uint32_t phase = 0;
-        int acc = 0;
-        uint32_t acc_phase = 0;
-        bool aborted = false;
-        for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-            for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
-                int ok = 1;
-                if (lane == 0)
-                    ok = wait_bounded(tempty(acc), acc_phase ^ 1u, &bars->abort, a.status);
-                ok = __shfl_sync(0xffffffffu, ok, 0);
-                if (!ok) {
-                    aborted = true;
-                    break;
-                }
-                ptx::tc_fence_after();
-                const uint32_t d_tmem = tmem + (uint32_t)(acc * kBN);
-                for (int kb = 0; kb < a.n_kb; ++kb) {
-                    ok = 1;
+        // ------------------------------------------------------------ MMA issuer (leader)
+        if (leader) {
+            constexpr uint32_t idesc = ptx::idesc_bf16_f32(kPairM, kBN);
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t acc_phase = 0;
+            bool aborted = false;
+            for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
+                for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
+                    int ok = 1;
                     if (lane == 0)
-                        ok = wait_bounded(full(stage), phase, &bars->abort, a.status);
+                        ok = wait_bounded<true>(tempty, acc_phase ^ 1u, &bars->abort, a.status);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (!ok) {
                         aborted = true;
                         break;
                     }
                     ptx::tc_fence_after();
-                    if (lane == 0) {
-                        const uint64_t da = ptx::sdesc_kmajor_sw128(sA(stage));
-                        const uint64_t db = ptx::sdesc_kmajor_sw128(sB(stage));
+                    for (int kb = 0; kb < a.n_kb; ++kb) {
+                        ok = 1;
+                        if (lane == 0)
+                            ok = wait_bounded(full(stage), phase, &bars->abort, a.status);
+                        ok = __shfl_sync(0xffffffffu, ok, 0);
+                        if (!ok) {
+                            aborted = true;
+                            break;
+                        }
+                        ptx::tc_fence_after();
+                        if (lane == 0) {
+                            const uint64_t da = ptx::sdesc_kmajor_sw128(sA(stage));
+                            const uint64_t db = ptx::sdesc_kmajor_sw128(sB(stage));
 #pragma unroll
-                        for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
-                            ptx::mma_bf16(d_tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
-                        ptx::mma_commit(empty(stage));
+                            for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
+                                ptx::mma_bf16_pair(tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
+                            ptx::mma_commit_pair_multicast(empty(stage), kBothCtas);
+                        }
+                        __syncwarp();
+                        if (++stage == kStages) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
                     }
+                    if (aborted)
+                        break;
+                    if (lane == 0)
+                        ptx::mma_commit_pair_multicast(tfull, kBothCtas);
                     __syncwarp();
-                    if (++stage == kStages) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
-                }
-                if (aborted)
-                    break;
-                if (lane == 0)
-                    ptx::mma_commit(tfull(acc));
-                __syncwarp();
-                if (++acc == 2) {
-                    acc = 0;
                     acc_phase ^= 1u;
                 }
             }
+            // No MMA may still be writing either CTA's TMEM when it is released.
+            if (lane == 0) {
+                ptx::mma_commit_pair(mma_done);
+                wait_drain(mma_done, 0);
+            }
+            __syncwarp();
         }
-        // No MMA may still be writing TMEM when it is released.
-        if (lane == 0) {
-            ptx::mma_commit(ptx::smem_u32(&bars->mma_done));
-            wait_drain(ptx::smem_u32(&bars->mma_done), 0);
-        }
-        __syncwarp();
     } else {
-        // ------------------------------------------------------------ epilogue (warps 2..5)
+        // ------------------------------------------------------------ epilogue (warps 2..5, both CTAs)
         const int q = warp & 3;  // this warp may only read TMEM lanes [32q, 32q + 32)
-        int acc = 0;
+        const uint32_t tempty_leader = ptx::mapa(tempty, 0);
         uint32_t acc_phase = 0;
         bool aborted = false;
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-            const int64_t row = (int64_t)mb * kBM + q * 32 + lane;
+            const int64_t row = (int64_t)mb * kPairM + (int)rank * kBM + q * 32 + lane;
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
             float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tl = 0.f;
             int32_t am = 0;
@@ -252,14 +267,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 const int nvalid = min(kBN, a.V - v0);
                 int ok = 1;
                 if (lane == 0)
-                    ok = wait_bounded(tfull(acc), acc_phase, &bars->abort, a.status);
+                    ok = wait_bounded(tfull, acc_phase, &bars->abort, a.status);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) {
                     aborted = true;
                     break;
                 }
                 ptx::tc_fence_after();
-                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
+                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
                 for (int c = 0; c < kBN / 32; ++c) {
                     const int cvalid = nvalid - c * 32;  // warp-uniform
@@ -307,40 +322,38 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                             tl = (j == tj) ? x[j] : tl;
                     }
                 }
-                // Accumulator fully read: hand it back to the MMA warp.
+                // Accumulator fully read by this warp: tell the leader's MMA warp.
                 ptx::tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
-                    ptx::mbar_arrive(tempty(acc));
-                if (++acc == 2) {
-                    acc = 0;
-                    acc_phase ^= 1u;
-                }
+                    ptx::mbar_arrive_cluster(tempty_leader);
+                acc_phase ^= 1u;
             }
             if (!aborted && row < a.N)
                 a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tl);
         }
-        ptx::tc_fence_before();
     }
 
+    // Neither CTA releases TMEM, or exits, while its peer may still use the pair's TMEM or barriers.
+    ptx::tc_fence_before();
     __syncthreads();
-    if (warp == 1) {
-        ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, kTmemCols);
-    }
+    ptx::cluster_sync();
+    ptx::tc_fence_after();
+    if (warp == 1)
+        ptx::tmem_dealloc_pair(tmem, kTmemCols);
 }
 
 }  // namespace
 
-// Choose the number of row-block groups: fewest tiles on the busiest CTA,
+// Choose the number of row-block groups: fewest tiles on the busiest pair,
 // then fewest passes over W (more groups = fewer passes).
-void score_schedule(int32_t n_mb, int32_t n_vt, int max_ctas, int32_t *n_groups, int32_t *G)
+void score_schedule(int32_t n_mb, int32_t n_vt, int max_units, int32_t *n_groups, int32_t *G)
 {
     int64_t best_rounds = -1;
     int32_t best_groups = 1, best_g = 1;
-    const int32_t top = n_mb < max_ctas ? n_mb : max_ctas;
+    const int32_t top = n_mb < max_units ? n_mb : max_units;
     for (int32_t groups = top; groups >= 1; --groups) {
-        int32_t g = max_ctas / groups;
+        int32_t g = max_units / groups;
         g = g < n_vt ? g : n_vt;
         g = g < kMaxRecordsPerRow ? g : kMaxRecordsPerRow;
         g = g < 1 ? 1 : g;
@@ -355,29 +368,60 @@ void score_schedule(int32_t n_mb, int32_t n_vt, int max_ctas, int32_t *n_groups,
     *G = best_g;
 }
 
-cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream)
+namespace {
+
+cudaLaunchConfig_t score_config(unsigned grid, cudaStream_t stream, cudaLaunchAttribute (&attr)[2])
 {
-    static thread_local int configured_device = -1;
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess)
-        return e;
-    if (configured_device != dev) {
-        e = cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScoreSmemBytes);
-        if (e != cudaSuccess)
-            return e;
-        configured_device = dev;
-    }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(a.n_groups * a.G));
+    cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kScoreThreads);
     cfg.dynamicSmemBytes = kScoreSmemBytes;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
+    return cfg;
+}
+
+// Per-device one-time set-up: shared-memory opt-in and the number of co-resident pairs.
+int configure_device()
+{
+    static int pairs[64];
+    static bool done[64];
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+        return -1;
+    if (!done[dev]) {
+        if (cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScoreSmemBytes) !=
+            cudaSuccess)
+            return -1;
+        cudaLaunchAttribute attr[2];
+        cudaLaunchConfig_t cfg = score_config(2, nullptr, attr);
+        cfg.numAttrs = 1;  // the cluster shape is what matters for the occupancy query
+        int clusters = 0;
+        if (cudaOccupancyMaxActiveClusters(&clusters, score_kernel, &cfg) != cudaSuccess || clusters < 1)
+            return -1;
+        pairs[dev] = clusters;
+        done[dev] = true;
+    }
+    return pairs[dev];
+}
+
+}  // namespace
+
+int score_max_pairs() { return configure_device(); }
+
+cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream)
+{
+    if (configure_device() < 1)
+        return cudaErrorUnknown;
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = score_config((unsigned)(2 * a.n_groups * a.G), stream, attr);
     return cudaLaunchKernelEx(&cfg, score_kernel, tmH, tmW, a);
 }
 

@@ -203,17 +203,20 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     CUtensorMap tmH, tmW;
     if ((rc = tensor_map(H, N, d, kBM, &tmH)) != WINO_OK)
         return rc;
-    if ((rc = tensor_map(W, V, d, kBN, &tmW)) != WINO_OK)
+    if ((rc = tensor_map(W, V, d, kHalfN, &tmW)) != WINO_OK)
         return rc;
+    const int max_pairs = score_max_pairs();
+    if (max_pairs < 1)
+        return WINO_ERR_CUDA;
     uint8_t *w8 = static_cast<uint8_t *>(ws);
     ScoreArgs a{};
     a.N = (int32_t)N;
     a.d = (int32_t)d;
     a.V = (int32_t)V;
-    a.n_mb = (int32_t)((N + kBM - 1) / kBM);
+    a.n_mb = (int32_t)((N + kPairM - 1) / kPairM);
     a.n_vt = (int32_t)((V + kBN - 1) / kBN);
     a.n_kb = (int32_t)((d + kBK - 1) / kBK);
-    score_schedule(a.n_mb, a.n_vt, info.sm_count, &a.n_groups, &a.G);
+    score_schedule(a.n_mb, a.n_vt, std::min(max_pairs, info.sm_count / 2), &a.n_groups, &a.G);
     a.ts = ts;
     a.part = reinterpret_cast<float4 *>(w8 + L.part);
     a.status = reinterpret_cast<int32_t *>(w8 + L.status);
