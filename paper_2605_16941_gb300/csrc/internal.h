@@ -14,7 +14,8 @@ namespace wino {
 // of H x 256 vocabulary columns.  Each CTA stages its own 128 rows of H and 128
 // of the 256 W rows per 64-wide K slice (128-byte swizzle rows) through a
 // 6-deep shared-memory ring, and holds its 128 rows x 256 columns of the fp32
-// accumulator in TMEM (one TMEM lane per row).
+// accumulator in TMEM (one TMEM lane per row), twice: the epilogue reads one
+// accumulator while the MMAs of the next tile fill the other.
 constexpr int kPairM = 256;  // rows per pair tile (UMMA M)
 constexpr int kBM = 128;     // rows per CTA
 constexpr int kBN = 256;     // vocabulary columns per tile (UMMA N)
@@ -26,7 +27,7 @@ constexpr uint32_t kStageBytesA = kBM * kBK * 2;     // 16 KB
 constexpr uint32_t kStageBytesB = kHalfN * kBK * 2;  // 16 KB
 constexpr uint32_t kRingBytes = kStages * (kStageBytesA + kStageBytesB);
 constexpr uint32_t kScoreSmemBytes = kRingBytes + 1024 /* alignment slack */ + 256 /* barriers */;
-constexpr uint32_t kTmemCols = kBN;  // one 256-column fp32 accumulator
+constexpr uint32_t kTmemCols = 2 * kBN;  // two 256-column fp32 accumulators: all 512 TMEM columns
 
 constexpr int kMaxBlkLen = 1024;
 

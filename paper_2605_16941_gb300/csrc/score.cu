@@ -15,12 +15,14 @@
 //   warp 0  TMA producer (both CTAs): streams 64-wide K slices of its 128 rows
 //           of H and of its 128 of the tile's 256 W rows into a 6-stage ring;
 //           both CTAs' copies complete on the LEADER's stage barrier;
-//   warp 1  TMEM allocation (both CTAs) and, in the leader only, the MMA
-//           issuer: 4 x (M256 N256 K16) per stage, committing stage release
-//           and accumulator-ready to both CTAs (multicast);
+//   warp 1  TMEM allocation (both CTAs, 512 columns = two 256-column fp32
+//           accumulators) and, in the leader only, the MMA issuer:
+//           4 x (M256 N256 K16) per stage, committing stage release and
+//           accumulator-ready to both CTAs (multicast);
 //   warps 2-5 epilogue (both CTAs): one thread per row (TMEM lane); online
-//           softmax over the tile's 256 columns, then release the
-//           accumulator to the leader's MMA warp (8 arrivals per tile).
+//           softmax over a tile's 256 columns while the MMAs of the next tile
+//           fill the other accumulator, then release the accumulator to the
+//           leader's MMA warp (8 arrivals per tile).
 // Work split: see ScoreArgs in internal.h.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA raises an
@@ -41,8 +43,8 @@ constexpr uint16_t kBothCtas = 0x3;
 struct alignas(8) Barriers {
     uint64_t full[kStages];   // leader: both CTAs' copies of a stage landed
     uint64_t empty[kStages];  // both: the stage's MMAs are done (multicast commit)
-    uint64_t tmem_full;       // both: the accumulator holds a finished tile (multicast commit)
-    uint64_t tmem_empty;      // leader: all 8 epilogue warps of the pair have read the accumulator
+    uint64_t tmem_full[2];    // both: accumulator i holds a finished tile (multicast commit)
+    uint64_t tmem_empty[2];   // leader: all 8 epilogue warps of the pair have read accumulator i
     uint64_t mma_done;        // leader: every MMA issued has completed
     uint32_t tmem_base;
     int32_t abort;
@@ -100,8 +102,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     auto sB = [&](int s) { return sA(s) + kStageBytesA; };
     auto full = [&](int s) { return ptx::smem_u32(&bars->full[s]); };
     auto empty = [&](int s) { return ptx::smem_u32(&bars->empty[s]); };
-    const uint32_t tfull = ptx::smem_u32(&bars->tmem_full);
-    const uint32_t tempty = ptx::smem_u32(&bars->tmem_empty);
+    auto tfull = [&](int i) { return ptx::smem_u32(&bars->tmem_full[i]); };
+    auto tempty = [&](int i) { return ptx::smem_u32(&bars->tmem_empty[i]); };
     const uint32_t mma_done = ptx::smem_u32(&bars->mma_done);
 
     // Set-up that touches no global memory overlaps the previous kernel (programmatic launch).
@@ -110,8 +112,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             ptx::mbar_init(full(s), 1);
             ptx::mbar_init(empty(s), 1);
         }
-        ptx::mbar_init(tfull, 1);
-        ptx::mbar_init(tempty, 8);  // 4 epilogue warps in each CTA of the pair
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(tfull(i), 1);
+            ptx::mbar_init(tempty(i), 8);  // 4 epilogue warps in each CTA of the pair
+        }
         ptx::mbar_init(mma_done, 1);
         bars->abort = 0;
         ptx::fence_barrier_init();
@@ -121,9 +125,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         ptx::prefetch_tensormap(&tmW);
     }
     if (warp == 1) {
-        // Both CTAs of the pair take part in the pair allocation.  256 columns: even if each CTA's
-        // request were served separately in both SMs, 2 x 256 fits the 512 columns of an SM, and the
-        // address check below then refuses to run.
+        // Both CTAs of the pair take part in the pair allocation, which reserves the same columns in
+        // both SMs; the address check below refuses to run if the two CTAs were given different ones.
         ptx::tmem_alloc_pair(ptx::smem_u32(&bars->tmem_base), kTmemCols);
         ptx::tmem_relinquish_pair();
     }
@@ -199,19 +202,21 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             constexpr uint32_t idesc = ptx::idesc_bf16_f32(kPairM, kBN);
             int stage = 0;
             uint32_t phase = 0;
+            int acc = 0;
             uint32_t acc_phase = 0;
             bool aborted = false;
             for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
                 for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
                     int ok = 1;
                     if (lane == 0)
-                        ok = wait_bounded<true>(tempty, acc_phase ^ 1u, &bars->abort, a.status);
+                        ok = wait_bounded<true>(tempty(acc), acc_phase ^ 1u, &bars->abort, a.status);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (!ok) {
                         aborted = true;
                         break;
                     }
                     ptx::tc_fence_after();
+                    const uint32_t d_tmem = tmem + (uint32_t)(acc * kBN);
                     for (int kb = 0; kb < a.n_kb; ++kb) {
                         ok = 1;
                         if (lane == 0)
@@ -227,7 +232,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                             const uint64_t db = ptx::sdesc_kmajor_sw128(sB(stage));
 #pragma unroll
                             for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
-                                ptx::mma_bf16_pair(tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
+                                ptx::mma_bf16_pair(d_tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
                             ptx::mma_commit_pair_multicast(empty(stage), kBothCtas);
                         }
                         __syncwarp();
@@ -239,9 +244,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                     if (aborted)
                         break;
                     if (lane == 0)
-                        ptx::mma_commit_pair_multicast(tfull, kBothCtas);
+                        ptx::mma_commit_pair_multicast(tfull(acc), kBothCtas);
                     __syncwarp();
-                    acc_phase ^= 1u;
+                    if (++acc == 2) {
+                        acc = 0;
+                        acc_phase ^= 1u;
+                    }
                 }
             }
             // No MMA may still be writing either CTA's TMEM when it is released.
@@ -254,7 +262,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     } else {
         // ------------------------------------------------------------ epilogue (warps 2..5, both CTAs)
         const int q = warp & 3;  // this warp may only read TMEM lanes [32q, 32q + 32)
-        const uint32_t tempty_leader = ptx::mapa(tempty, 0);
+        int acc = 0;
         uint32_t acc_phase = 0;
         bool aborted = false;
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
@@ -267,14 +275,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 const int nvalid = min(kBN, a.V - v0);
                 int ok = 1;
                 if (lane == 0)
-                    ok = wait_bounded(tfull, acc_phase, &bars->abort, a.status);
+                    ok = wait_bounded(tfull(acc), acc_phase, &bars->abort, a.status);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) {
                     aborted = true;
                     break;
                 }
                 ptx::tc_fence_after();
-                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
 #pragma unroll 1
                 for (int c = 0; c < kBN / 32; ++c) {
                     const int cvalid = nvalid - c * 32;  // warp-uniform
@@ -326,8 +334,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 ptx::tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
-                    ptx::mbar_arrive_cluster(tempty_leader);
-                acc_phase ^= 1u;
+                    ptx::mbar_arrive_cluster(ptx::mapa(tempty(acc), 0));
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
             }
             if (!aborted && row < a.N)
                 a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tl);
