@@ -22,7 +22,11 @@
  *     current-block row of position l, kind 1 = its shadow-block row; row
  *     index n = (2*s + kind)*blk_len + l, N = 2*n_seq*blk_len.
  *   - `stream` is a cudaStream_t (NULL = legacy default stream); all work is
- *     enqueued on it asynchronously, in order.
+ *     enqueued on it asynchronously, in order.  Consecutive WINO calls on one
+ *     stream overlap (programmatic dependent launch): a call may start reading
+ *     its H and W while the previous WINO call's last kernel is finishing, so
+ *     H and W must not be memory that the previous call writes (its tokens,
+ *     counts, flags, statistics or workspace).
  *   - Return value: WINO_OK (0) or a negative wino_status.  On an argument
  *     error nothing is enqueued.  Device-side failures (a bounded wait that
  *     expired) are reported in the workspace status word, see

@@ -217,31 +217,28 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
 #pragma unroll
             for (int i = 0; i < kRec; ++i) {
                 const int j = lane + 32 * i;
-                r[i] = (j < a.G) ? __ldcg(pr + j) : make_float4(-INFINITY, 0.f, __int_as_float(INT32_MAX), 0.f);
+                r[i] = (j < a.G) ? __ldcg(pr + j) : make_float4(-INFINITY, 0.f, __int_as_float(INT32_MAX), -INFINITY);
             }
-            int32_t t = -1;
-            float tl = 0.f;
-            if (lane == 0) {
-                t = row_target(a.ts, row, a.V);
-                if (t >= 0)
-                    tl = __ldcg(pr + (t / kBN) % a.G).w;
-            }
-            float m = -INFINITY, s = 0.f;
+            // The record of the pair whose tiles hold the row's target carries its logit; the others -inf.
+            float m = -INFINITY, s = 0.f, tl = -INFINITY;
             int32_t idx = INT32_MAX;
 #pragma unroll
-            for (int i = 0; i < kRec; ++i)
+            for (int i = 0; i < kRec; ++i) {
                 combine(m, s, idx, r[i].x, r[i].y, __float_as_int(r[i].z));
+                tl = fmaxf(tl, r[i].w);
+            }
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) {
                 const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
                 const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
                 const int32_t i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+                tl = fmaxf(tl, __shfl_xor_sync(0xffffffffu, tl, off));
                 combine(m, s, idx, m2, s2, i2);
             }
             if (lane == 0) {
                 a.argmax[row] = idx;
                 a.pmax[row] = 1.0f / s;
-                a.ptarget[row] = (t >= 0) ? ptx::ex2((tl - m) * kLog2e) / s : 0.0f;
+                a.ptarget[row] = (tl > -INFINITY) ? ptx::ex2((tl - m) * kLog2e) / s : 0.0f;
                 __threadfence();  // publish this row before the CTA signals its ticket
             }
         }

@@ -66,7 +66,7 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
 constexpr int kMaxRecordsPerRow = 256;
 
 // Partial record: running max logit m, sum of exp(l - m), argmax (int bits),
-// logit of the row's target if the target lies in one of the CTA's tiles (else 0).
+// logit of the row's target if the target lies in one of the pair's tiles (else -inf).
 struct ScoreArgs {
     int32_t N, d, V;
     int32_t n_mb, n_vt, n_kb;  // n_mb: 256-row blocks

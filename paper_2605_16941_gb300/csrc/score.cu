@@ -137,20 +137,27 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const uint32_t peer_tmem = ptx::ld_shared_cluster_u32(ptx::mapa(ptx::smem_u32(&bars->tmem_base), rank ^ 1u));
     const bool tmem_ok = (peer_tmem == tmem);
 
-    // From here on global memory is read and written: wait for the grid before us.
-    ptx::grid_dep_wait();
+    // Programmatic launch: the TMA producer and the MMA warp only read H and W, which the grid before
+    // us (the finish kernel of the previous WINO call on this stream) never writes, so they start at
+    // once.  Everything that touches what that grid reads or writes -- the token state (targets), the
+    // partial records, the status word and the tickets -- waits for it (grid_dep_wait) first.
     ptx::grid_dep_launch_dependents();
-    if (blockIdx.x == 0 && threadIdx.x == 0)
-        *a.status = tmem_ok ? WINO_OK : WINO_ERR_UNSUPPORTED;
-    for (int i = blockIdx.x * kScoreThreads + threadIdx.x; i < a.n_tickets; i += gridDim.x * kScoreThreads)
-        a.tickets[i] = 0;
 
     const int grp = pair % a.n_groups;  // 256-row blocks grp, grp + n_groups, ...
     const int col = pair / a.n_groups;  // vocabulary tiles col, col + G, ...
 
-    if (!tmem_ok) {
-        if (threadIdx.x == 0)
+    if (warp >= 2 || !tmem_ok) {
+        ptx::grid_dep_wait();
+        if (blockIdx.x == 0 && threadIdx.x == 64)
+            *a.status = tmem_ok ? WINO_OK : WINO_ERR_UNSUPPORTED;
+        if (!tmem_ok && threadIdx.x == 64)
             atomicExch(a.status, (int32_t)WINO_ERR_UNSUPPORTED);
+        for (int i = blockIdx.x * 128 + (int)threadIdx.x - 64; i < a.n_tickets; i += gridDim.x * 128)
+            if (threadIdx.x >= 64)
+                a.tickets[i] = 0;
+    }
+    if (!tmem_ok) {
+        // nothing to do: the status word reports the failed allocation check
     } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer (both CTAs)
         const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every vocabulary tile
@@ -268,7 +275,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
             const int64_t row = (int64_t)mb * kPairM + (int)rank * kBM + q * 32 + lane;
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
-            float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tl = 0.f;
+            float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tl = -INFINITY;
             int32_t am = 0;
             for (int vt = col; vt < a.n_vt; vt += a.G) {
                 const int32_t v0 = vt * kBN;
