@@ -16,6 +16,8 @@ SHAPES = [
     (257, 128, 513),
     (128, 4096, 2048),
     (384, 520, 777),
+    (100, 64, 19400),   # last pair: one 256-wide tile with 200 valid columns
+    (256, 128, 50000),  # several 256-wide tiles per pair and a 128-wide tail tile
 ]
 
 
