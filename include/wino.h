@@ -141,6 +141,32 @@ WINO_API int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t 
               int32_t *counts, int8_t *flags, void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * wino_step without a caller-supplied workspace, for callers that cannot
+ * allocate device memory: an inference-server plugin that is handed only its
+ * input and output buffers, a process whose memory pool owns all device
+ * memory, or a decode loop that must not call cudaMalloc / cudaFree while it
+ * runs (both synchronise the device).  (The paper has no counterpart: this is
+ * an interface choice of this library.)
+ *
+ * Same arguments, kernels and results as wino_step, with the workspace taken
+ * from one fixed array of WINO_STATIC_SCRATCH_BYTES in device memory that the
+ * library reserves on every GPU that loads it, until the process exits.  The
+ * call allocates nothing.  Problems whose wino_workspace_size exceeds the
+ * array are rejected with WINO_ERR_WORKSPACE before anything is launched
+ * (for V >= 32768, any d: N = 2 * n_seq * blk_len up to 4080 rows).
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * Every call on a device shares the one array: calls that may overlap on the
+ * GPU (different streams, or host threads without ordering) race and must be
+ * serialised by the caller.  The kernels clear the words they rely on (status
+ * word, tickets) at the start of each call, so the array needs no
+ * initialisation; the per-row statistics it holds are not returned.
+ */
+#define WINO_STATIC_SCRATCH_BYTES (16u << 20)
+WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens,
+                                      const wino_params *p, int32_t *counts, int8_t *flags, void *stream);
+
+/*
  * Waits for `stream`, then reads the workspace status word written by the
  * last score launch that used `ws`: WINO_OK, or WINO_ERR_DEVICE_TIMEOUT.
  */

@@ -9,16 +9,16 @@ transformer: the LM-head GEMM fused with a full-vocabulary online softmax,
 the cross-tile merge, and the in-place state update, as CUDA kernels behind
 a C ABI (``include/wino.h``).  The Python side marshals arguments only.
 """
-from ._abi import (EXPORTS, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_DRAFT_IS_MASK, FLAG_NONE, FLAG_REMASK,
+from ._abi import (EXPORTS, WINO_STATIC_SCRATCH_BYTES, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_DRAFT_IS_MASK, FLAG_NONE, FLAG_REMASK,
                    WINO_ERR_ARG, WINO_ERR_CUDA, WINO_ERR_DEVICE_TIMEOUT, WINO_ERR_MAX_STEPS, WINO_ERR_SHAPE,
                    WINO_ERR_UNSUPPORTED, WINO_ERR_WORKSPACE, WINO_OK, WINO_OPT_FREEZE_FINISHED, WinoError, WinoParams, lib, library_path,
-                   make_params, wino_draft_verify, wino_profile_begin, wino_profile_end, wino_read_device_status, wino_score_rows, wino_status_string,
+                   make_params, wino_draft_verify, wino_profile_begin, wino_profile_end, wino_read_device_status, wino_score_rows, wino_status_string, wino_step_static_scratch,
                    wino_step, wino_version, wino_workspace_size, workspace)
 
 __all__ = [
-    "EXPORTS", "FLAG_DRAFT", "FLAG_DRAFT_FALLBACK", "FLAG_DRAFT_IS_MASK", "FLAG_NONE", "FLAG_REMASK",
+    "EXPORTS", "WINO_STATIC_SCRATCH_BYTES", "FLAG_DRAFT", "FLAG_DRAFT_FALLBACK", "FLAG_DRAFT_IS_MASK", "FLAG_NONE", "FLAG_REMASK",
     "WINO_ERR_ARG", "WINO_ERR_CUDA", "WINO_ERR_DEVICE_TIMEOUT", "WINO_ERR_MAX_STEPS", "WINO_ERR_SHAPE",
     "WINO_ERR_UNSUPPORTED", "WINO_ERR_WORKSPACE", "WINO_OK", "WINO_OPT_FREEZE_FINISHED", "WinoError", "WinoParams", "lib", "library_path",
-    "make_params", "wino_draft_verify", "wino_profile_begin", "wino_profile_end", "wino_read_device_status", "wino_score_rows", "wino_status_string",
+    "make_params", "wino_draft_verify", "wino_profile_begin", "wino_profile_end", "wino_read_device_status", "wino_score_rows", "wino_status_string", "wino_step_static_scratch",
     "wino_step", "wino_version", "wino_workspace_size", "workspace",
 ]

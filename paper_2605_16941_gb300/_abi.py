@@ -30,8 +30,11 @@ FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0,
 WINO_OPT_FREEZE_FINISHED = 1
 
 EXPORTS = ("wino_workspace_size", "wino_score_rows", "wino_draft_verify", "wino_step",
-           "wino_read_device_status", "wino_profile_begin", "wino_profile_end", "wino_status_string",
-           "wino_version")
+           "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
+           "wino_status_string", "wino_version")
+
+# size of the fixed device array behind wino_step_static_scratch
+WINO_STATIC_SCRATCH_BYTES = 16 << 20
 
 
 class WinoError(RuntimeError):
@@ -66,6 +69,8 @@ def lib() -> C.CDLL:
         L.wino_draft_verify.argtypes = [vp, vp, vp, vp, C.POINTER(WinoParams), vp, vp, vp]
         L.wino_step.restype = C.c_int
         L.wino_step.argtypes = [vp, vp, i64, i64, vp, C.POINTER(WinoParams), vp, vp, vp, sz, vp]
+        L.wino_step_static_scratch.restype = C.c_int
+        L.wino_step_static_scratch.argtypes = [vp, vp, i64, i64, vp, C.POINTER(WinoParams), vp, vp, vp]
         L.wino_read_device_status.restype = C.c_int
         L.wino_read_device_status.argtypes = [vp, vp, C.POINTER(C.c_int)]
         L.wino_profile_begin.restype = C.c_int
@@ -153,6 +158,15 @@ def wino_step(H, W, tokens, params: WinoParams, counts, ws, flags=None, stream=N
     ws_bytes = ws.numel() * ws.element_size()
     _check(lib().wino_step(_ptr(H), _ptr(W), d, V, _ptr(tokens), C.byref(params), _ptr(counts), _ptr(flags),
                            _ptr(ws), ws_bytes, _stream(stream)), "wino_step")
+
+
+def wino_step_static_scratch(H, W, tokens, params: WinoParams, counts, flags=None, stream=None, *,
+                             d: int | None = None, V: int | None = None) -> None:
+    """wino_step with the library's fixed device scratch instead of a caller workspace (allocates nothing)."""
+    d = int(H.shape[1]) if d is None else d
+    V = int(W.shape[0]) if V is None else V
+    _check(lib().wino_step_static_scratch(_ptr(H), _ptr(W), d, V, _ptr(tokens), C.byref(params), _ptr(counts),
+                                          _ptr(flags), _stream(stream)), "wino_step_static_scratch")
 
 
 def wino_read_device_status(ws, stream=None) -> int:
