@@ -118,6 +118,22 @@ class ClockSampler:
                 "samples": len(sm), "samples_in_timed_region": len(inside)}
 
 
+def ncu_traffic(workload_name: str):
+    """DRAM bytes per score launch from the committed ncu capture, if it was taken on this workload and
+    the score kernel's source has not changed since (else None)."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "score_kernel_traffic.txt")) as f:
+            rec = json.load(f)
+        with open(os.path.join(ROOT, "paper_2605_16941_gb300", "csrc", "score.cu"), "rb") as f:
+            h = hashlib.sha256(f.read()).hexdigest()[:16]
+    except (OSError, ValueError):
+        return None
+    if rec.get("workload") != workload_name or rec.get("score_cu_sha256_prefix") != h:
+        return None
+    return float(rec["dram_bytes_read"]) + float(rec["dram_bytes_write"])
+
+
 def gpu_uuid(dev):
     import torch
     try:
@@ -344,7 +360,7 @@ def run_wino(args, rank, world, local_rank):
         "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_dict(w),
         "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
-                     "traffic": None, "kernel": "score_kernel (fused LM-head GEMM + online vocab softmax)",
+                     "traffic": ncu_traffic(w.name), "kernel": "score_kernel (fused LM-head GEMM + online vocab softmax)",
                      "algorithmic_per_launch": {"bytes": alg_bytes, "flops": flops},
                      "avg_launch_us": score_avg_s * 1e6, "launches_timed": score_n, "peak_source": peak_src,
                      "timing": "per-launch CUDA events around the score kernel over a second region of K steps",
