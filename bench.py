@@ -134,6 +134,21 @@ def ncu_traffic(workload_name: str):
     return float(rec["dram_bytes_read"]) + float(rec["dram_bytes_write"])
 
 
+def job_time_max(seconds_local: float, world: int, device=None) -> float:
+    """The slowest rank's time (max over ranks); the job's throughput divides all ranks' work by it."""
+    import torch
+    t = torch.tensor([seconds_local], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rows_per_s(rows_per_rank_step: int, steps: int, world: int, t_max_s: float) -> float:
+    """Whole-job scored rows/s: every rank decodes its own replica (weak scaling)."""
+    return world * rows_per_rank_step * steps / t_max_s
+
+
 def gpu_uuid(dev):
     import torch
     try:
@@ -288,10 +303,7 @@ def run_wino(args, rank, world, local_rank):
         clocks.stop()
     if wino.wino_read_device_status(wsp, stream=sid) != wino.WINO_OK:
         raise RuntimeError("device status not OK after the timed region")
-    t_max = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
-    t_max = float(t_max.item())
+    t_max = 1e3 * job_time_max(elapsed_ms / 1e3, world, device=dev)
 
     # ---- end to end through the C ABI with host buffers (pinned), one host read of the result per step
     Hh = [torch.from_numpy(np.ascontiguousarray(h).view(np.int16)).pin_memory() for h in Hs]
@@ -319,10 +331,7 @@ def run_wino(args, rank, world, local_rank):
         e2e_step(i)
     torch.cuda.synchronize(dev)
     te = time.perf_counter() - te0
-    te_t = torch.tensor([te], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(te_t, op=dist.ReduceOp.MAX)
-    te = float(te_t.item())
+    te = job_time_max(te, world, device=dev)
     h2d = Hh[0].numel() * 2 + tok_h.numel() * 4
     d2h = tok_out.numel() * 4 + cnt_out.numel() * 4
 
@@ -346,7 +355,7 @@ def run_wino(args, rank, world, local_rank):
     else:
         achieved, peak, unit = flops / score_avg_s / 1e12, peaks["bf16_tflops"], "TFLOP/s"
     step_s = t_max / 1e3 / args.steps
-    value = world * w.N * args.steps / (t_max / 1e3)
+    value = job_rows_per_s(w.N, args.steps, world, t_max / 1e3)
     clock_info = clocks.summary(tw0, tw1) if clocks else None
 
     cpu = None
@@ -370,7 +379,7 @@ def run_wino(args, rank, world, local_rank):
                                                                                       peaks["bf16_tflops"])},
         "step_roofline_frac": max(t_flop, w_bytes / (peaks["hbm_gbs"] * 1e9)) / step_s,
         "tflops_per_step": flops / step_s / 1e12,
-        "e2e": {"value": world * w.N * e2e_steps / te, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job_rows_per_s(w.N, e2e_steps, world, te), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * te / e2e_steps},
         "gpu_launches": 2 * args.steps,
         "clocks": clock_info,
