@@ -72,6 +72,12 @@ typedef struct {
     int32_t blk_len;   /* L_b, 1..1024; blk_start + blk_len <= seq_len                           */
     int32_t max_steps; /* step budget for loop drivers; unused by the calls below               */
     int32_t options;   /* bit set of WINO_OPT_* below; 0 = plain Eq. 4 on every sequence        */
+    int32_t step_index;   /* k, the index of the state this step produces (Y^(k)); see last_change */
+    int32_t *last_change; /* optional device int32 [n_seq, seq_len]: every position whose token the
+                             step changes gets step_index.  Started at 0 and carried through a whole
+                             decode with step_index = 1, 2, ..., it ends as each position's WINO
+                             finalization step t_l = min{t : y_l^(j) = y_l^final for all j >= t}
+                             (Sec. 5.1; 0 for the prompt).  NULL: not recorded. */
 } wino_params;
 
 /*

@@ -177,12 +177,14 @@ int oracle_row_targets(const int32_t *tokens, int64_t n_seq, int64_t seq_len, in
  * in the block}; flags[s * blk_len + l] (optional) gets the outcome codes.
  * With freeze_finished != 0, a sequence whose block has no MASK is not
  * stepped at all: the loop "until no MASK is left" (Sec. 4.2.3) has ended
- * for it.
+ * for it.  If last_change (int32 [n_seq, seq_len]) is given, every position
+ * whose token this step changes is set to step_index.
  */
 int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t blk_start,
                         int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                         const int32_t *argmax, const double *pmax, const double *ptarget,
-                        int32_t *counts, int8_t *flags, int freeze_finished)
+                        int32_t *counts, int8_t *flags, int freeze_finished, int32_t step_index,
+                        int32_t *last_change)
 {
     if (!tokens || !argmax || !pmax || !ptarget || !counts || n_seq < 0 || blk_len < 1 ||
         blk_start < 0 || blk_start + blk_len > seq_len)
@@ -228,6 +230,7 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
         int32_t drafted = 0, remasked = 0, left = 0;
         for (int64_t l = 0; l < blk_len; ++l) {
             int8_t code = 0;
+            int32_t before = y[l];
             if (inD[l]) {
                 y[l] = argmax[row_blk + l];
                 if (y[l] == mask_id)
@@ -242,6 +245,8 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
                 ++remasked;
             }
             left += (y[l] == mask_id);
+            if (last_change && y[l] != before)
+                last_change[s * seq_len + blk_start + l] = step_index;
             if (flags)
                 flags[s * blk_len + l] = code;
         }
@@ -264,7 +269,7 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
 int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, int64_t n_seq,
                 int64_t seq_len, int64_t blk_start, int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                 int32_t *counts, int8_t *flags, int32_t *argmax_out, double *pmax_out, double *ptarget_out,
-                double *gap_out, int nthreads, int freeze_finished)
+                double *gap_out, int nthreads, int freeze_finished, int32_t step_index, int32_t *last_change)
 {
     const int64_t N = n_seq * 2 * blk_len;
     int32_t *target = (int32_t *)malloc((size_t)N * sizeof(int32_t));
@@ -279,7 +284,7 @@ int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int3
             rc = oracle_score_rows(H, W, N, d, V, target, am, pm, pt, gp, NULL, NULL, nthreads);
         if (rc == ORACLE_OK)
             rc = oracle_draft_verify(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, tau1, tau2, am, pm,
-                                     pt, counts, flags, freeze_finished);
+                                     pt, counts, flags, freeze_finished, step_index, last_change);
         if (rc == ORACLE_OK) {
             if (argmax_out)
                 memcpy(argmax_out, am, (size_t)N * sizeof(int32_t));

@@ -46,7 +46,8 @@ class WinoError(RuntimeError):
 class WinoParams(C.Structure):
     _fields_ = [("tau1", C.c_float), ("tau2", C.c_float), ("mask_id", C.c_int32), ("n_seq", C.c_int32),
                 ("seq_len", C.c_int32), ("blk_start", C.c_int32), ("blk_len", C.c_int32),
-                ("max_steps", C.c_int32), ("options", C.c_int32)]
+                ("max_steps", C.c_int32), ("options", C.c_int32), ("step_index", C.c_int32),
+                ("last_change", C.c_void_p)]
 
 
 def library_path() -> Path:
@@ -128,9 +129,10 @@ def workspace(N: int, d: int, V: int, device=None):
 
 
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
-                max_steps: int = 4096, freeze_finished: bool = False) -> WinoParams:
+                max_steps: int = 4096, freeze_finished: bool = False, step_index: int = 0,
+                last_change=None) -> WinoParams:
     return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps,
-                      WINO_OPT_FREEZE_FINISHED if freeze_finished else 0)
+                      WINO_OPT_FREEZE_FINISHED if freeze_finished else 0, step_index, _ptr(last_change))
 
 
 def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, N: int | None = None,

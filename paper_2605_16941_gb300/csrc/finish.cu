@@ -162,8 +162,11 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
             next = mask;
             code = 3;
         }
-        if (next != prev)
+        if (next != prev) {
             y[l] = next;
+            if (p.last_change)  // WINO finalization step bookkeeping (Sec. 5.1)
+                p.last_change[(int64_t)s * p.seq_len + p.blk_start + l] = p.step_index;
+        }
         drafted += (code == 1 || code == 2);
         remasked += (code == 3);
         left += (next == mask);

@@ -37,12 +37,15 @@ class LoopStats:
 
 def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float, mask_id: int,
            hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
-           on_step: Callable | None = None) -> LoopStats:
+           on_step: Callable | None = None, last_change=None) -> LoopStats:
     """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
 
     ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
-    for global step ``k``.  ``on_step(k, blk_start, counts_host, flags)`` is called
-    after every step (for tests and statistics).
+    for global step ``k`` (0-based; the step produces state Y^(k+1)).  ``on_step(k,
+    blk_start, counts_host, flags)`` is called after every step (for tests and
+    statistics).  ``last_change`` (device int32 [n_seq, S], zeros at the start)
+    receives, per position, the last step that changed it: after the decode, each
+    position's WINO finalization step t_l (Sec. 5.1).
     """
     import torch
 
@@ -58,12 +61,14 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     k = 0
     for b in range(n_blocks):
         b0 = prompt_len + b * blk_len
-        p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True)
+        p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True,
+                        last_change=last_change)
         bs = BlockStats(block=b, blk_start=b0)
         while True:
             if bs.steps >= max_steps:
                 raise WinoError(WINO_ERR_MAX_STEPS, f"decode: block {b} not finished after {max_steps} steps")
             H = hidden(k, b0)
+            p.step_index = k + 1
             wino_step(H, W, tokens, p, counts, ws, flags=flags, stream=stream)
             counts_host.copy_(counts, non_blocking=True)
             torch.cuda.current_stream(dev).synchronize() if stream is None else stream.synchronize()

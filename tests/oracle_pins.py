@@ -350,7 +350,50 @@ def pin_freeze_finished(O):
     assert tok.tolist() == [[1, M, M, 4], [1, 6, M, M]] and cnt.tolist() == [[0, 2, 2], [1, 2, 2]], (tok, cnt)
 
 
-EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_only_draft_never_remasks, pin_greedy_reduction,
+def finalization_steps_from_trajectory(traj):
+    """t_l = min{t : y_l^(j) = y_l^(K) for all j >= t} over a trajectory Y^(0..K) (Sec. 5.1)."""
+    Y = np.stack(traj)  # [K + 1, n_seq, S]
+    final = Y[-1]
+    differs = Y != final[None]
+    K = Y.shape[0] - 1
+    # the last index j at which the state still differs from the final one, plus one; 0 if never
+    any_diff = differs.any(0)
+    last_diff = K - np.argmax(differs[::-1], axis=0)
+    return np.where(any_diff, last_diff + 1, 0).astype(np.int32)
+
+
+def pin_finalization_steps(O):
+    """The step bookkeeping equals the paper's finalization step computed from the whole trajectory,
+    including positions that were drafted, re-masked and drafted again."""
+    w = ws.Workload("pin_final", d=64, V=500, n_seq=3, blk_len=8, bias=((1.0, 0.0, 5.0),), n_blocks=2,
+                    bias_step=0.4, tau1=0.6, tau2=0.9)
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    tokens = st.tokens.copy()
+    last = np.zeros_like(tokens)
+    traj = [tokens.copy()]
+    k = 0
+    remasked = 0
+    for blk in range(w.n_blocks):
+        b0 = w.block_start(blk)
+        st.blk_start = b0
+        for _ in range(400):
+            H = ws.hidden_states(w, W, st, step=k)
+            k += 1
+            r = O.step(H, W, tokens, b0, w.blk_len, w.mask_id, w.tau1, w.tau2, freeze_finished=True, step_index=k,
+                       last_change=last)
+            tokens = r.tokens
+            traj.append(tokens.copy())
+            remasked += int(r.counts[:, 1].sum())
+            if np.all(r.counts[:, 2] == 0):
+                break
+    assert remasked > 0, "the trajectory should revoke some tokens"
+    want = finalization_steps_from_trajectory(traj)
+    assert np.array_equal(last, want), (last, want)
+    assert np.all(last[:, :w.prompt_len] == 0) and np.all(last[:, w.prompt_len:] >= 1)
+
+
+EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_finalization_steps, pin_only_draft_never_remasks, pin_greedy_reduction,
             pin_eq4_exhaustive_properties, pin_loop_terminates]
 
 ALL_PINS = SCORING_PINS + EQ4_PINS

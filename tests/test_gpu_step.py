@@ -38,17 +38,22 @@ def test_draft_verify_bit_exact(n_seq, L, S, b0, taus, freeze):
     if freeze and n_seq > 1:
         tokens[0, b0:b0 + L] = rng.integers(0, M, size=L)  # a finished block
     t1, t2 = taus
+    last0 = rng.integers(0, 5, size=(n_seq, S)).astype(np.int32)
+    ref_last = last0.copy()
     ref_tok, ref_cnt, ref_fl = oracle.draft_verify(tokens, b0, L, M, f32(t1), f32(t2), am, pm.astype(np.float64),
-                                                   pt.astype(np.float64), freeze_finished=freeze)
+                                                   pt.astype(np.float64), freeze_finished=freeze, step_index=7,
+                                                   last_change=ref_last)
     tok_d = dev(tokens)
+    last_d = dev(last0)
     counts = torch.full((n_seq, 3), -9, dtype=torch.int32, device="cuda")
     flags = torch.full((n_seq, L), -9, dtype=torch.int8, device="cuda")
-    p = wino.make_params(t1, t2, M, n_seq, S, b0, L, freeze_finished=freeze)
+    p = wino.make_params(t1, t2, M, n_seq, S, b0, L, freeze_finished=freeze, step_index=7, last_change=last_d)
     wino.wino_draft_verify(tok_d, dev(am), dev(pm), dev(pt), p, counts, flags)
     torch.cuda.synchronize()
     assert np.array_equal(host(tok_d), ref_tok)
     assert np.array_equal(host(counts), ref_cnt)
     assert np.array_equal(host(flags), ref_fl)
+    assert np.array_equal(host(last_d), ref_last)
 
 
 def _gpu_step(w, Wd, tokens, H, blk_start, tau1=None):
@@ -176,28 +181,38 @@ def test_decode_loop_tiny_lockstep():
     Wd = dev(W)
     st = ws.initial_state(w)
     tok_d = dev(st.tokens)
+    last_d = torch.zeros_like(tok_d)
     record = {}
+    traj = [st.tokens.copy()]
 
     def hidden(k, b0):
         st.blk_start = b0
         H = ws.hidden_states(w, W, st, step=k)
         record["pre"] = host(tok_d).copy()
+        record["last_pre"] = host(last_d).copy()
         record["H"] = H
         return dev(H)
 
     reports = []
 
     def on_step(k, b0, counts, flags):
+        last_ref = record["last_pre"]
         o = oracle.step(record["H"], W, record["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2,
-                        freeze_finished=True)
-        reports.append(compare_step(record["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1,
-                                    w.tau2))
+                        freeze_finished=True, step_index=k + 1, last_change=last_ref)
+        rep = compare_step(record["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1, w.tau2)
+        if rep["flagged_positions"] == 0:  # same decisions: the finalization bookkeeping must agree exactly
+            assert np.array_equal(host(last_d), last_ref)
+        reports.append(rep)
+        traj.append(host(tok_d).copy())
 
     stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
-                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=500)
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=500,
+                        last_change=last_d)
     final = host(tok_d)
     assert not np.any(final[:, w.prompt_len:] == w.mask_id)
     assert np.array_equal(final[:, :w.prompt_len], st.tokens[:, :w.prompt_len])
+    from oracle_pins import finalization_steps_from_trajectory
+    assert np.array_equal(host(last_d), finalization_steps_from_trajectory(traj))  # t_l of Sec. 5.1
     print("tiny loop steps/block", [b.steps for b in stats.blocks], "flagged",
           sum(r["flagged_positions"] for r in reports))
 

@@ -42,6 +42,9 @@ MUTANTS = [
     ("left_counts_old_state", "left += (y[l] == mask_id);", "left += (prev[l] == mask_id);"),
     ("freeze_ignored", "if (freeze_finished && n_mask == 0) {", "if (0) {"),
     ("freeze_always", "if (freeze_finished && n_mask == 0) {", "if (n_mask == 0) {"),
+    ("last_change_on_every_position", "if (last_change && y[l] != before)", "if (last_change)"),
+    ("last_change_off_by_one", "last_change[s * seq_len + blk_start + l] = step_index;",
+     "last_change[s * seq_len + blk_start + l] = step_index - 1;"),
 ]
 
 
