@@ -90,6 +90,16 @@ typedef struct {
 #define WINO_OPT_FREEZE_FINISHED 1
 
 /*
+ * WINO_OPT_NO_SHADOW: WINO+ inference (Sec. 5.3, Sec. 6.1.2).  The model was
+ * trained to follow WINO's order, so decoding drops the shadow block and
+ * verification: each sequence contributes only its blk_len block rows (row
+ * index s*blk_len + l, N = n_seq*blk_len), a masked position is drafted iff
+ * its confidence exceeds tau1 (the single threshold; the at-least-one rule
+ * still applies), and nothing is re-masked (tau2 is ignored).
+ */
+#define WINO_OPT_NO_SHADOW 2
+
+/*
  * Bytes of scratch the score path needs for N rows of dimension d over a
  * vocabulary of V entries (per-tile partial softmax statistics, targets and
  * per-row results, plus one status word).  `ws` passed to wino_score_rows /
@@ -121,7 +131,9 @@ WINO_API int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, in
  * Eq. 4 on every sequence's current block, in place on tokens[n_seq, seq_len]
  * (int32), from per-row statistics in [s][kind][l] order (argmax/pmax of the
  * kind-0 rows drive drafting; ptarget of the kind-1 rows, i.e. the
- * probability of the position's CURRENT token, drives verification).
+ * probability of the position's CURRENT token, drives verification).  With
+ * WINO_OPT_NO_SHADOW the rows are [s][l] block rows only and ptarget may be
+ * NULL.
  *   counts [n_seq, 3] int32 out: {drafted (MASK -> token), re-masked,
  *                                MASKs left in the block after the step}
  *   flags  [n_seq, blk_len] int8 out or NULL: per position 0 unchanged,
@@ -139,7 +151,8 @@ WINO_API int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const flo
  * (the current token of each decoded position, none for masked positions and
  * for block rows), every row is scored as in wino_score_rows, and Eq. 4 is
  * applied as in wino_draft_verify.
- *   H [2*n_seq*blk_len, d] bf16 rows in [s][kind][l] order; W [V, d] bf16.
+ *   H [2*n_seq*blk_len, d] bf16 rows in [s][kind][l] order (with
+ *     WINO_OPT_NO_SHADOW: [n_seq*blk_len, d], block rows only); W [V, d] bf16.
  * If a device wait expired, tokens are left unchanged and every counts entry
  * is set to WINO_ERR_DEVICE_TIMEOUT.
  */

@@ -72,11 +72,11 @@ class Oracle:
         L.oracle_row_targets.restype = C.c_int
         L.oracle_row_targets.argtypes = [vp, i64, i64, i64, i64, i32, vp]
         L.oracle_draft_verify.restype = C.c_int
-        L.oracle_draft_verify.argtypes = [vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp, C.c_int, i32,
-                                          vp]
+        L.oracle_draft_verify.argtypes = [vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp, C.c_int,
+                                          C.c_int, i32, vp]
         L.oracle_step.restype = C.c_int
         L.oracle_step.argtypes = [vp, vp, i64, i64, vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp,
-                                  vp, C.c_int, C.c_int, i32, vp]
+                                  vp, C.c_int, C.c_int, C.c_int, i32, vp]
         L.oracle_num_threads.restype = C.c_int
         L.oracle_num_threads.argtypes = []
         self.L = L
@@ -123,31 +123,35 @@ class Oracle:
 
     def draft_verify(self, tokens: np.ndarray, blk_start: int, blk_len: int, mask_id: int, tau1: float,
                      tau2: float, argmax: np.ndarray, pmax: np.ndarray, ptarget: np.ndarray,
-                     freeze_finished: bool = False, step_index: int = 0, last_change: np.ndarray | None = None):
+                     freeze_finished: bool = False, step_index: int = 0, last_change: np.ndarray | None = None,
+                     no_shadow: bool = False):
         """Eq. 4 on a copy of ``tokens``; returns (new_tokens, counts [n_seq,3], flags [n_seq, blk_len]).
-        ``last_change`` (int32 [n_seq, seq_len], updated in place) gets ``step_index`` where a token changes."""
+        ``last_change`` (int32 [n_seq, seq_len], updated in place) gets ``step_index`` where a token changes.
+        ``no_shadow``: WINO+ inference, rows are block rows only and ``ptarget`` may be None."""
         tok = np.array(tokens, dtype=np.int32, copy=True, order="C")
         n_seq, S = tok.shape
-        N = n_seq * 2 * blk_len
-        am, pm, pt = _c(argmax, np.int32), _c(pmax, np.float64), _c(ptarget, np.float64)
-        assert am.shape == pm.shape == pt.shape == (N,)
+        N = n_seq * (1 if no_shadow else 2) * blk_len
+        am, pm = _c(argmax, np.int32), _c(pmax, np.float64)
+        pt = None if ptarget is None else _c(ptarget, np.float64)
+        assert am.shape == pm.shape == (N,) and (pt is None or pt.shape == (N,))
         counts = np.empty((n_seq, 3), np.int32)
         flags = np.empty((n_seq, blk_len), np.int8)
         rc = self.L.oracle_draft_verify(_p(tok), n_seq, S, blk_start, blk_len, mask_id, float(tau1),
                                         float(tau2), _p(am), _p(pm), _p(pt), _p(counts), _p(flags),
-                                        int(bool(freeze_finished)), int(step_index), _p(_lc(last_change, tok)))
+                                        int(bool(freeze_finished)), int(bool(no_shadow)), int(step_index),
+                                        _p(_lc(last_change, tok)))
         if rc != 0:
             raise RuntimeError(f"oracle_draft_verify failed: {rc}")
         return tok, counts, flags
 
     def step(self, H_bits: np.ndarray, W_bits: np.ndarray, tokens: np.ndarray, blk_start: int, blk_len: int,
              mask_id: int, tau1: float, tau2: float, nthreads: int = 0, freeze_finished: bool = False,
-             step_index: int = 0, last_change: np.ndarray | None = None) -> StepResult:
-        """One whole WINO step on a copy of ``tokens`` (``last_change`` as in draft_verify)."""
+             step_index: int = 0, last_change: np.ndarray | None = None, no_shadow: bool = False) -> StepResult:
+        """One whole WINO step on a copy of ``tokens`` (``last_change``, ``no_shadow`` as in draft_verify)."""
         H, W = _c(H_bits, np.uint16), _c(W_bits, np.uint16)
         tok = np.array(tokens, dtype=np.int32, copy=True, order="C")
         n_seq, S = tok.shape
-        N = n_seq * 2 * blk_len
+        N = n_seq * (1 if no_shadow else 2) * blk_len
         V, d = W.shape
         assert H.shape == (N, d)
         r = StepResult(tok, np.empty((n_seq, 3), np.int32), np.empty((n_seq, blk_len), np.int8),
@@ -155,8 +159,8 @@ class Oracle:
                        np.empty(N, np.float64))
         rc = self.L.oracle_step(_p(H), _p(W), d, V, _p(tok), n_seq, S, blk_start, blk_len, mask_id, float(tau1),
                                 float(tau2), _p(r.counts), _p(r.flags), _p(r.argmax), _p(r.pmax), _p(r.ptarget),
-                                _p(r.gap), nthreads, int(bool(freeze_finished)), int(step_index),
-                                _p(_lc(last_change, tok)))
+                                _p(r.gap), nthreads, int(bool(freeze_finished)), int(bool(no_shadow)),
+                                int(step_index), _p(_lc(last_change, tok)))
         if rc != 0:
             raise RuntimeError(f"oracle_step failed: {rc}")
         return r
@@ -193,12 +197,12 @@ def row_targets(tokens, blk_start: int, blk_len: int, mask_id: int):
 
 
 def draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget, freeze_finished=False,
-                 step_index=0, last_change=None):
+                 step_index=0, last_change=None, no_shadow=False):
     return default().draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget,
-                                  freeze_finished, step_index, last_change)
+                                  freeze_finished, step_index, last_change, no_shadow)
 
 
 def step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads: int = 0,
-         freeze_finished: bool = False, step_index: int = 0, last_change=None) -> StepResult:
+         freeze_finished: bool = False, step_index: int = 0, last_change=None, no_shadow: bool = False) -> StepResult:
     return default().step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads, freeze_finished,
-                          step_index, last_change)
+                          step_index, last_change, no_shadow)

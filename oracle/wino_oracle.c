@@ -179,14 +179,19 @@ int oracle_row_targets(const int32_t *tokens, int64_t n_seq, int64_t seq_len, in
  * stepped at all: the loop "until no MASK is left" (Sec. 4.2.3) has ended
  * for it.  If last_change (int32 [n_seq, seq_len]) is given, every position
  * whose token this step changes is set to step_index.
+ *
+ * no_shadow != 0 is WINO+ inference (Sec. 5.3, Sec. 6.1.2): there is no
+ * shadow block, the rows are the block rows only ([s][l], row s*blk_len + l),
+ * drafting uses the single threshold tau1 with the same at-least-one rule,
+ * and R is empty (ptarget may be NULL).
  */
 int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t blk_start,
                         int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                         const int32_t *argmax, const double *pmax, const double *ptarget,
-                        int32_t *counts, int8_t *flags, int freeze_finished, int32_t step_index,
+                        int32_t *counts, int8_t *flags, int freeze_finished, int no_shadow, int32_t step_index,
                         int32_t *last_change)
 {
-    if (!tokens || !argmax || !pmax || !ptarget || !counts || n_seq < 0 || blk_len < 1 ||
+    if (!tokens || !argmax || !pmax || (!ptarget && !no_shadow) || !counts || n_seq < 0 || blk_len < 1 ||
         blk_start < 0 || blk_start + blk_len > seq_len)
         return ORACLE_ERR_ARG;
     int32_t *prev = (int32_t *)malloc((size_t)blk_len * sizeof(int32_t));
@@ -200,13 +205,13 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
     }
     for (int64_t s = 0; s < n_seq; ++s) {
         int32_t *y = tokens + s * seq_len + blk_start;
-        const int64_t row_blk = (s * 2 + 0) * blk_len; /* kind 0: Y_cur rows  */
-        const int64_t row_shd = (s * 2 + 1) * blk_len; /* kind 1: Y_shad rows */
+        const int64_t row_blk = no_shadow ? s * blk_len : (s * 2 + 0) * blk_len; /* kind 0: Y_cur rows  */
+        const int64_t row_shd = (s * 2 + 1) * blk_len;                           /* kind 1: Y_shad rows */
         int64_t n_draft = 0, n_mask = 0;
         for (int64_t l = 0; l < blk_len; ++l) {
             prev[l] = y[l];
             inD[l] = (prev[l] == mask_id) && (pmax[row_blk + l] > tau1);
-            inR[l] = (prev[l] != mask_id) && (ptarget[row_shd + l] < tau2);
+            inR[l] = !no_shadow && (prev[l] != mask_id) && (ptarget[row_shd + l] < tau2);
             n_draft += inD[l];
             n_mask += (prev[l] == mask_id);
         }
@@ -269,9 +274,10 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
 int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, int64_t n_seq,
                 int64_t seq_len, int64_t blk_start, int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                 int32_t *counts, int8_t *flags, int32_t *argmax_out, double *pmax_out, double *ptarget_out,
-                double *gap_out, int nthreads, int freeze_finished, int32_t step_index, int32_t *last_change)
+                double *gap_out, int nthreads, int freeze_finished, int no_shadow, int32_t step_index,
+                int32_t *last_change)
 {
-    const int64_t N = n_seq * 2 * blk_len;
+    const int64_t N = n_seq * (no_shadow ? 1 : 2) * blk_len;
     int32_t *target = (int32_t *)malloc((size_t)N * sizeof(int32_t));
     int32_t *am = (int32_t *)malloc((size_t)N * sizeof(int32_t));
     double *pm = (double *)malloc((size_t)N * sizeof(double));
@@ -279,12 +285,18 @@ int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int3
     double *gp = (double *)malloc((size_t)N * sizeof(double));
     int rc = ORACLE_ERR_NOMEM;
     if (target && am && pm && pt && gp) {
-        rc = oracle_row_targets(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, target);
+        if (no_shadow) {  /* block rows only: no row has a target */
+            for (int64_t n = 0; n < N; ++n)
+                target[n] = -1;
+            rc = ORACLE_OK;
+        } else {
+            rc = oracle_row_targets(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, target);
+        }
         if (rc == ORACLE_OK)
             rc = oracle_score_rows(H, W, N, d, V, target, am, pm, pt, gp, NULL, NULL, nthreads);
         if (rc == ORACLE_OK)
             rc = oracle_draft_verify(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, tau1, tau2, am, pm,
-                                     pt, counts, flags, freeze_finished, step_index, last_change);
+                                     pt, counts, flags, freeze_finished, no_shadow, step_index, last_change);
         if (rc == ORACLE_OK) {
             if (argmax_out)
                 memcpy(argmax_out, am, (size_t)N * sizeof(int32_t));

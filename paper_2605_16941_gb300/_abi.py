@@ -28,6 +28,7 @@ FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0,
 
 # wino_params.options
 WINO_OPT_FREEZE_FINISHED = 1
+WINO_OPT_NO_SHADOW = 2
 
 EXPORTS = ("wino_workspace_size", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
@@ -130,9 +131,10 @@ def workspace(N: int, d: int, V: int, device=None):
 
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
                 max_steps: int = 4096, freeze_finished: bool = False, step_index: int = 0,
-                last_change=None) -> WinoParams:
-    return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps,
-                      WINO_OPT_FREEZE_FINISHED if freeze_finished else 0, step_index, _ptr(last_change))
+                last_change=None, no_shadow: bool = False) -> WinoParams:
+    opts = (WINO_OPT_FREEZE_FINISHED if freeze_finished else 0) | (WINO_OPT_NO_SHADOW if no_shadow else 0)
+    return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps, opts, step_index,
+                      _ptr(last_change))
 
 
 def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, N: int | None = None,

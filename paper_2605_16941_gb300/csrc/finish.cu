@@ -70,9 +70,10 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
     }
     const int L = p.blk_len;
     const int32_t mask = p.mask_id;
+    const bool shadow = !(p.options & WINO_OPT_NO_SHADOW);  // WINO+ inference has no verification rows
     int32_t *y = tokens + (int64_t)s * p.seq_len + p.blk_start;
-    const int64_t rb = (int64_t)(2 * s) * L;      // kind-0 rows: the block Y_cur
-    const int64_t rs = (int64_t)(2 * s + 1) * L;  // kind-1 rows: the shadow block Y_shad
+    const int64_t rb = (int64_t)(shadow ? 2 * s : s) * L;  // kind-0 rows: the block Y_cur
+    const int64_t rs = (int64_t)(2 * s + 1) * L;           // kind-1 rows: the shadow block Y_shad
 
     int32_t yv[kPer], av[kPer];
     float pm[kPer], pt[kPer];
@@ -83,7 +84,7 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
             yv[i] = y[l];
             av[i] = __ldcg(argmax + rb + l);
             pm[i] = __ldcg(pmax + rb + l);
-            pt[i] = __ldcg(ptarget + rs + l);
+            pt[i] = shadow ? __ldcg(ptarget + rs + l) : 1.0f;  // 1.0 is never below tau2 <= 1: no re-mask
         }
     }
     // Pass 1: how many masked positions clear tau1, and the most confident masked position.
@@ -158,7 +159,7 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
                 next = av[i];
                 code = (next == mask) ? 4 : (l == fallback ? 2 : 1);
             }
-        } else if (pt[i] < p.tau2) {
+        } else if (shadow && pt[i] < p.tau2) {
             next = mask;
             code = 3;
         }
@@ -253,7 +254,7 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
     __syncthreads();
     if (threadIdx.x == 0) {
         int32_t nd = 0;
-        const int64_t per_seq = 2 * (int64_t)a.p.blk_len;
+        const int64_t per_seq = ((a.p.options & WINO_OPT_NO_SHADOW) ? 1 : 2) * (int64_t)a.p.blk_len;
         const int64_t rend = min(row0 + kFinishRows, (int64_t)a.N);
         for (int64_t r = row0; r < rend;) {
             const int64_t sq = r / per_seq;

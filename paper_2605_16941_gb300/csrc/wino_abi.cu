@@ -300,7 +300,7 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
 int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream)
 {
-    if (!tokens || !argmax || !pmax || !ptarget || !counts)
+    if (!tokens || !argmax || !pmax || !counts || !p || (!ptarget && !(p->options & WINO_OPT_NO_SHADOW)))
         return WINO_ERR_ARG;
     int rc = check_params(p);
     if (rc != WINO_OK)
@@ -324,7 +324,8 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     int rc = check_params(p);
     if (rc != WINO_OK)
         return rc;
-    const int64_t N = (int64_t)p->n_seq * 2 * p->blk_len;
+    const bool shadow = !(p->options & WINO_OPT_NO_SHADOW);
+    const int64_t N = (int64_t)p->n_seq * (shadow ? 2 : 1) * p->blk_len;
     if (!shape_ok(N, d, V) || p->mask_id >= V)
         return WINO_ERR_SHAPE;
     const WsLayout L = ws_layout(N, V);
@@ -335,7 +336,7 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     float *pm = reinterpret_cast<float *>(w8 + L.pmax);
     float *pt = reinterpret_cast<float *>(w8 + L.ptarget);
     TargetSource ts{};
-    ts.tokens = tokens;
+    ts.tokens = shadow ? tokens : nullptr;  // only shadow rows have targets
     ts.seq_len = p->seq_len;
     ts.blk_start = p->blk_start;
     ts.blk_len = p->blk_len;

@@ -393,7 +393,29 @@ def pin_finalization_steps(O):
     assert np.all(last[:, :w.prompt_len] == 0) and np.all(last[:, w.prompt_len:] >= 1)
 
 
-EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_finalization_steps, pin_only_draft_never_remasks, pin_greedy_reduction,
+def pin_no_shadow_is_threshold_decoding(O):
+    """WINO+ inference (no shadow block): on the block rows it is exactly Eq. 4 with verification off
+    (tau2 = 0, the "only draft" ablation of Sec. 6.3.4), whatever the shadow rows would have said."""
+    rng = np.random.default_rng(23)
+    n_seq, L, M, P = 40, 12, 70, 5
+    for tau1 in (0.25, 0.5, 1.0):
+        tokens = rng.integers(0, M + 1, size=(n_seq, P + L + 3)).astype(np.int32)
+        tokens[rng.random(tokens.shape) < 0.5] = M
+        am_b = rng.integers(0, M + 1, size=(n_seq, L)).astype(np.int32)
+        pm_b = np.round(rng.random((n_seq, L)) * 8) / 8
+        # WINO+ rows: [s][l]
+        t1, c1, f1 = O.draft_verify(tokens, P, L, M, tau1, 0.9, am_b.reshape(-1), pm_b.reshape(-1), None,
+                                    no_shadow=True)
+        # the same block rows inside the [s][kind][l] layout, shadow rows random, tau2 = 0
+        am = np.stack([am_b, rng.integers(0, M, size=(n_seq, L))], 1).reshape(-1).astype(np.int32)
+        pm = np.stack([pm_b, rng.random((n_seq, L))], 1).reshape(-1)
+        pt = rng.random(2 * n_seq * L)
+        t2, c2, f2 = O.draft_verify(tokens, P, L, M, tau1, 0.0, am, pm, pt)
+        assert np.array_equal(t1, t2) and np.array_equal(c1, c2) and np.array_equal(f1, f2)
+        assert np.all(c1[:, 1] == 0)
+
+
+EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_finalization_steps, pin_no_shadow_is_threshold_decoding, pin_only_draft_never_remasks, pin_greedy_reduction,
             pin_eq4_exhaustive_properties, pin_loop_terminates]
 
 ALL_PINS = SCORING_PINS + EQ4_PINS

@@ -269,3 +269,75 @@ def test_decode_loop_b16():
     print("loop_b16 steps/block", [b.steps for b in stats.blocks], "total", stats.total_steps,
           "drafted/block", [b.drafted for b in stats.blocks], "remasked/block", [b.remasked for b in stats.blocks],
           "oracle-checked steps", checked)
+
+
+@pytest.mark.parametrize("n_seq,L,S,b0", CASES[:5], ids=[f"B{c[0]}_L{c[1]}" for c in CASES[:5]])
+def test_draft_verify_no_shadow_bit_exact(n_seq, L, S, b0):
+    """WINO+ inference rule (block rows only, single threshold, no re-mask), ptarget not passed."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, f32, host
+    M = 997
+    rng = np.random.default_rng(n_seq * 77 + L)
+    tokens, _, _, _ = _random_case(rng, n_seq, L, S, b0, M)
+    N = n_seq * L
+    am = rng.integers(0, M + 1, size=N).astype(np.int32)
+    pm = rng.random(N).astype(np.float32)
+    pm[rng.random(N) < 0.05] = np.float32(0.75)
+    for tau in (0.5, 0.75, 1.0):
+        ref_tok, ref_cnt, ref_fl = oracle.draft_verify(tokens, b0, L, M, f32(tau), f32(0.9), am,
+                                                       pm.astype(np.float64), None, no_shadow=True)
+        tok_d = dev(tokens)
+        counts = torch.full((n_seq, 3), -9, dtype=torch.int32, device="cuda")
+        flags = torch.full((n_seq, L), -9, dtype=torch.int8, device="cuda")
+        p = wino.make_params(tau, 0.9, M, n_seq, S, b0, L, no_shadow=True)
+        wino.wino_draft_verify(tok_d, dev(am), dev(pm), None, p, counts, flags)
+        torch.cuda.synchronize()
+        assert np.array_equal(host(tok_d), ref_tok)
+        assert np.array_equal(host(counts), ref_cnt) and np.array_equal(host(flags), ref_fl)
+        assert np.all(ref_cnt[:, 1] == 0)
+
+
+def test_decode_loop_wino_plus_lockstep():
+    """WINO+ inference decode (no shadow block, one threshold) through the loop driver, every step
+    re-run by the oracle from the same state; finalization steps tracked as well."""
+    import dataclasses
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import compare_step, dev, host
+    w = ws.Workload("wino_plus_loop", d=128, V=3000, n_seq=3, blk_len=32, bias=((1.0, 0.0, 8.0),), n_blocks=2,
+                    bias_step=0.4, tau1=0.8, tau2=0.9, shadow=False)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    tok_d = dev(st.tokens)
+    last_d = torch.zeros_like(tok_d)
+    rec = {}
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        H = ws.hidden_states(w, W, st, step=k)
+        assert H.shape[0] == w.n_seq * w.blk_len
+        rec["pre"], rec["H"], rec["last"] = host(tok_d).copy(), H, host(last_d).copy()
+        return dev(H)
+
+    reports = []
+
+    def on_step(k, b0, counts, flags):
+        o = oracle.step(rec["H"], W, rec["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2, freeze_finished=True,
+                        step_index=k + 1, last_change=rec["last"], no_shadow=True)
+        ow = dataclasses.replace(o)  # compare_step reads the [s][kind][l] layout: give it block rows twice
+        ow.pmax = np.repeat(o.pmax.reshape(w.n_seq, 1, w.blk_len), 2, axis=1).reshape(-1)
+        ow.gap = np.repeat(o.gap.reshape(w.n_seq, 1, w.blk_len), 2, axis=1).reshape(-1)
+        ow.ptarget = np.ones(2 * w.N)  # never below tau2: no verification decision to flag
+        rep = compare_step(rec["pre"], host(tok_d), counts, ow, b0, w.blk_len, w.mask_id, w.tau1, w.tau2)
+        assert rep["remasked"] == 0
+        if rep["flagged_positions"] == 0:
+            assert np.array_equal(host(last_d), rec["last"])
+        reports.append(rep)
+
+    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=500,
+                        last_change=last_d, no_shadow=True)
+    final = host(tok_d)
+    assert not np.any(final[:, w.prompt_len:] == w.mask_id)
+    assert all(b.remasked == 0 for b in stats.blocks)
+    print("WINO+ loop steps/block", [b.steps for b in stats.blocks])

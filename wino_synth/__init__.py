@@ -109,6 +109,7 @@ class Workload:
     seed: int = 0
     hold: float = 0.0  # fraction of pre-decoded positions that hold their planted target
     bias_step: float = 0.0  # growth of every component's upper bound per global step
+    shadow: bool = True  # False: WINO+ inference, block rows only (no verification rows)
 
     @property
     def mask_id(self) -> int:
@@ -123,8 +124,12 @@ class Workload:
         return self.prompt_len + self.gen_len
 
     @property
+    def kinds(self) -> int:
+        return 2 if self.shadow else 1
+
+    @property
     def N(self) -> int:
-        return self.n_seq * 2 * self.blk_len
+        return self.n_seq * self.kinds * self.blk_len
 
     def block_start(self, block: int = 0) -> int:
         return self.prompt_len + block * self.blk_len
@@ -204,15 +209,16 @@ def row_biases(w: Workload, step: int = 0) -> np.ndarray:
 def hidden_states(w: Workload, W: np.ndarray, state: State, step: int = 0) -> np.ndarray:
     """H[N, d] bf16 bits for the current block of ``state`` at global step ``step``.
 
-    Rows are ``[s][kind][l]``; both kinds of position l plant target
-    ``state.targets[s, blk_start - prompt_len + l]`` with independent noise and bias."""
+    Rows are ``[s][kind][l]`` (``[s][l]`` without the shadow block); every row of
+    position l plants target ``state.targets[s, blk_start - prompt_len + l]`` with
+    independent noise and bias."""
     z = _normal_rows_bf16(w.N, w.d, 1.0, [w.seed, _TAG_H, step])  # noise (bf16-exact values)
     h = bf16_bits_to_f32(z).reshape(w.N, w.d)
     b = row_biases(w, step)
     gen0 = state.blk_start - w.prompt_len
     L = w.blk_len
     t = state.targets[:, gen0: gen0 + L]  # [n_seq, L]
-    t_rows = np.repeat(t[:, None, :], 2, axis=1).reshape(-1)  # [s][kind][l]
+    t_rows = np.repeat(t[:, None, :], w.kinds, axis=1).reshape(-1)  # [s][kind][l]
     wt = bf16_bits_to_f32(W[t_rows])  # [N, d]
     nrm2 = np.einsum("nd,nd->n", wt.astype(np.float64), wt.astype(np.float64)).astype(np.float32)
     h += (b / nrm2)[:, None] * wt
@@ -223,4 +229,4 @@ def row_targets_planted(w: Workload, state: State) -> np.ndarray:
     """Planted target token of every hidden-state row (int32 [N]); for reporting."""
     gen0 = state.blk_start - w.prompt_len
     t = state.targets[:, gen0: gen0 + w.blk_len]
-    return np.repeat(t[:, None, :], 2, axis=1).reshape(-1).astype(np.int32)
+    return np.repeat(t[:, None, :], w.kinds, axis=1).reshape(-1).astype(np.int32)
