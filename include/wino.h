@@ -119,13 +119,16 @@ WINO_API int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
  *   argmax  [N] int32 out: argmax_v l_v, the smallest v among exact ties
  *   pmax    [N] float out: max_v p_v = 1 / sum_v exp(l_v - max_u l_u)
  *   ptarget [N] float out: p_target, 0 where the row has no target
+ *   entropy [N] float out or NULL: H(p) = -sum_v p_v ln p_v, the per-row
+ *           quantity WINO+'s deferral and sharpening terms use (Sec. 5.3,
+ *           Eq. 6-7); NULL skips it (the decode path never computes it)
  * Shapes: 1 <= N <= 2^24, 8 <= d <= 65536 with d % 8 == 0, 2 <= V <= 2^27.
  * Logits are accumulated in fp32 on the tensor cores; the softmax runs in
  * fp32.  The status word in `ws` is cleared at the start of the call.
  */
 WINO_API int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V,
-                    const int32_t *target, int32_t *argmax, float *pmax, float *ptarget, void *ws,
-                    size_t ws_bytes, void *stream);
+                    const int32_t *target, int32_t *argmax, float *pmax, float *ptarget, float *entropy,
+                    void *ws, size_t ws_bytes, void *stream);
 
 /*
  * Eq. 4 on every sequence's current block, in place on tokens[n_seq, seq_len]
@@ -172,7 +175,7 @@ WINO_API int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t 
  * library reserves on every GPU that loads it, until the process exits.  The
  * call allocates nothing.  Problems whose wino_workspace_size exceeds the
  * array are rejected with WINO_ERR_WORKSPACE before anything is launched
- * (for V >= 32768, any d: N = 2 * n_seq * blk_len up to 4080 rows).
+ * (for V >= 32768, any d: N = 2 * n_seq * blk_len up to 3266 rows).
  * The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress); make that first call before any stream capture.
  * Every call on a device shares the one array: calls that may overlap on the

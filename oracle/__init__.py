@@ -44,6 +44,7 @@ class RowStats:
     gap: np.ndarray  # float64 [N] top-1 minus top-2 logit
     maxlogit: np.ndarray  # float64 [N]
     logz: np.ndarray  # float64 [N]
+    entropy: np.ndarray  # float64 [N], -sum p log p
 
 
 @dataclass
@@ -68,7 +69,7 @@ class Oracle:
         L.oracle_logits_row.restype = None
         L.oracle_logits_row.argtypes = [vp, vp, i64, i64, vp]
         L.oracle_score_rows.restype = C.c_int
-        L.oracle_score_rows.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, vp, vp, vp, vp, C.c_int]
+        L.oracle_score_rows.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, vp, vp, vp, vp, vp, C.c_int]
         L.oracle_row_targets.restype = C.c_int
         L.oracle_row_targets.argtypes = [vp, i64, i64, i64, i64, i32, vp]
         L.oracle_draft_verify.restype = C.c_int
@@ -105,9 +106,10 @@ class Oracle:
         t = None if target is None else _c(target, np.int32)
         if t is not None:
             assert t.shape == (N,)
-        out = RowStats(np.empty(N, np.int32), *(np.empty(N, np.float64) for _ in range(5)))
+        out = RowStats(np.empty(N, np.int32), *(np.empty(N, np.float64) for _ in range(6)))
         rc = self.L.oracle_score_rows(_p(H), _p(W), N, d, V, _p(t), _p(out.argmax), _p(out.pmax),
-                                      _p(out.ptarget), _p(out.gap), _p(out.maxlogit), _p(out.logz), nthreads)
+                                      _p(out.ptarget), _p(out.gap), _p(out.maxlogit), _p(out.logz),
+                                      _p(out.entropy), nthreads)
         if rc != 0:
             raise RuntimeError(f"oracle_score_rows failed: {rc}")
         return out

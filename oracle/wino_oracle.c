@@ -79,11 +79,13 @@ void oracle_logits_row(const uint16_t *h, const uint16_t *W, int64_t d, int64_t 
  *   gap[n]     = m - (largest logit over v != argmax[n]); 0 on an exact tie
  *   maxlogit[n]= m            (optional output, may be NULL)
  *   logz[n]    = m + log Z    (optional output, may be NULL)
+ *   entropy[n] = -sum_v p_v log p_v, the entropy WINO+'s deferral and
+ *                sharpening terms use (Sec. 5.3, Eq. 6-7) (optional, may be NULL)
  * Rows are independent; they are spread over nthreads (<= 0: library default).
  */
 int oracle_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V,
                       const int32_t *target, int32_t *argmax, double *pmax, double *ptarget,
-                      double *gap, double *maxlogit, double *logz, int nthreads)
+                      double *gap, double *maxlogit, double *logz, double *entropy, int nthreads)
 {
     if (!H || !W || !argmax || !pmax || !ptarget || !gap || N < 0 || d < 1 || V < 1)
         return ORACLE_ERR_ARG;
@@ -131,6 +133,15 @@ int oracle_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d
                 maxlogit[n] = m;
             if (logz)
                 logz[n] = m + log(Z);
+            if (entropy) {
+                double h = 0.0;
+                for (int64_t v = 0; v < V; ++v) {
+                    const double p = exp(logit[v] - m) / Z;
+                    if (p > 0.0)
+                        h -= p * log(p);
+                }
+                entropy[n] = h;
+            }
         }
         free(logit);
     }
@@ -293,7 +304,7 @@ int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int3
             rc = oracle_row_targets(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, target);
         }
         if (rc == ORACLE_OK)
-            rc = oracle_score_rows(H, W, N, d, V, target, am, pm, pt, gp, NULL, NULL, nthreads);
+            rc = oracle_score_rows(H, W, N, d, V, target, am, pm, pt, gp, NULL, NULL, NULL, nthreads);
         if (rc == ORACLE_OK)
             rc = oracle_draft_verify(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, tau1, tau2, am, pm,
                                      pt, counts, flags, freeze_finished, no_shadow, step_index, last_change);

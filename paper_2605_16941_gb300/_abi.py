@@ -66,7 +66,7 @@ def lib() -> C.CDLL:
         L.wino_workspace_size.restype = C.c_int
         L.wino_workspace_size.argtypes = [i64, i64, i64, C.POINTER(sz)]
         L.wino_score_rows.restype = C.c_int
-        L.wino_score_rows.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, vp, vp, sz, vp]
+        L.wino_score_rows.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, vp, vp, vp, sz, vp]
         L.wino_draft_verify.restype = C.c_int
         L.wino_draft_verify.argtypes = [vp, vp, vp, vp, C.POINTER(WinoParams), vp, vp, vp]
         L.wino_step.restype = C.c_int
@@ -137,15 +137,16 @@ def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int
                       _ptr(last_change))
 
 
-def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, N: int | None = None,
+def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, entropy=None, N: int | None = None,
                     d: int | None = None, V: int | None = None) -> None:
-    """Fused LM-head + full-vocabulary softmax statistics; shapes default to H.shape / W.shape."""
+    """Fused LM-head + full-vocabulary softmax statistics (and, given ``entropy``, H(p) per row);
+    shapes default to H.shape / W.shape."""
     N = int(H.shape[0]) if N is None else N
     d = int(H.shape[1]) if d is None else d
     V = int(W.shape[0]) if V is None else V
     ws_bytes = ws.numel() * ws.element_size()
     _check(lib().wino_score_rows(_ptr(H), _ptr(W), N, d, V, _ptr(target), _ptr(argmax), _ptr(pmax), _ptr(ptarget),
-                                 _ptr(ws), ws_bytes, _stream(stream)), "wino_score_rows")
+                                 _ptr(entropy), _ptr(ws), ws_bytes, _stream(stream)), "wino_score_rows")
 
 
 def wino_draft_verify(tokens, argmax, pmax, ptarget, params: WinoParams, counts, flags=None, stream=None) -> None:

@@ -6,7 +6,9 @@
 //   argmax   = smallest vocabulary id among the maximal logits,
 //   pmax     = max_v p_v = 1 / sum_v exp(l_v - m),
 //   ptarget  = p_target = exp(l_t - m) / sum_v exp(l_v - m)    (0 without a target),
-// the three statistics Eq. 2 and Eq. 3 use.  In a whole step (wino_step) every
+// the three statistics Eq. 2 and Eq. 3 use, and on request the entropy
+//   H(p)     = -sum_v p_v log p_v = ln Z - sum_v exp(l_v - m) (l_v - m) / Z
+// that WINO+'s deferral and sharpening terms use (Sec. 5.3, Eq. 6-7).  In a whole step (wino_step) every
 // CTA then adds its merged rows to its sequences' tickets; the CTA that
 // completes a sequence's 2*L_b rows applies Eq. 4 to that sequence, so merge
 // and update need one launch.  Tickets are cleared by the score kernel of the
@@ -34,6 +36,7 @@ namespace wino {
 namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kFinishRows = 8;  // rows (warps) per finish CTA; also the CTA size of the Eq. 4 kernels
 
 // Fold (m2, s2, i2) into (m, s, i): the larger max wins, the smaller index on equal maxima.
@@ -46,6 +49,29 @@ __device__ __forceinline__ void combine(float &m, float &s, int32_t &i, float m2
         i = i2;
     m = M;
     s = a + b;
+}
+
+// As combine, also folding u = sum exp(l - m) (l - m) log2(e) (rescaled to the new max like s).
+__device__ __forceinline__ void combine_u(float &m, float &s, float &u, int32_t &i, float m2, float s2, float u2,
+                                          int32_t i2)
+{
+    const float M = fmaxf(m, m2);
+    float a = 0.f, b = 0.f, ua = 0.f, ub = 0.f;
+    if (m != -INFINITY) {
+        const float al = ptx::ex2((m - M) * kLog2e);
+        a = s * al;
+        ua = al * fmaf((m - M) * kLog2e, s, u);
+    }
+    if (m2 != -INFINITY) {
+        const float bl = ptx::ex2((m2 - M) * kLog2e);
+        b = s2 * bl;
+        ub = bl * fmaf((m2 - M) * kLog2e, s2, u2);
+    }
+    if (m2 > m || (m2 == m && i2 < i))
+        i = i2;
+    m = M;
+    s = a + b;
+    u = ua + ub;
 }
 
 // Block-wide reduction scratch for eq4_block.
@@ -212,6 +238,8 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
                 a.argmax[row] = -1;
                 a.pmax[row] = __int_as_float(0x7fc00000);
                 a.ptarget[row] = __int_as_float(0x7fc00000);
+                if (a.entropy)
+                    a.entropy[row] = __int_as_float(0x7fc00000);
             }
         } else {
             const float4 *pr = a.part + row * a.G;
@@ -224,25 +252,47 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
                 r[i] = (j < a.G) ? __ldcg(pr + j) : make_float4(-INFINITY, 0.f, __int_as_float(INT32_MAX), -INFINITY);
             }
             // The record of the pair whose tiles hold the row's target carries its logit; the others -inf.
-            float m = -INFINITY, s = 0.f, tl = -INFINITY;
+            float m = -INFINITY, s = 0.f, tl = -INFINITY, u = 0.f;
             int32_t idx = INT32_MAX;
+            if (!a.entropy) {
 #pragma unroll
-            for (int i = 0; i < kRec; ++i) {
-                combine(m, s, idx, r[i].x, r[i].y, __float_as_int(r[i].z));
-                tl = fmaxf(tl, r[i].w);
-            }
+                for (int i = 0; i < kRec; ++i) {
+                    combine(m, s, idx, r[i].x, r[i].y, __float_as_int(r[i].z));
+                    tl = fmaxf(tl, r[i].w);
+                }
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-                const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
-                const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
-                const int32_t i2 = __shfl_xor_sync(0xffffffffu, idx, off);
-                tl = fmaxf(tl, __shfl_xor_sync(0xffffffffu, tl, off));
-                combine(m, s, idx, m2, s2, i2);
+                for (int off = 16; off > 0; off >>= 1) {
+                    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+                    const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+                    const int32_t i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+                    tl = fmaxf(tl, __shfl_xor_sync(0xffffffffu, tl, off));
+                    combine(m, s, idx, m2, s2, i2);
+                }
+            } else {
+                const float *pu = a.part_u + row * a.G;
+#pragma unroll
+                for (int i = 0; i < kRec; ++i) {
+                    const int j = lane + 32 * i;
+                    combine_u(m, s, u, idx, r[i].x, r[i].y, (j < a.G) ? __ldcg(pu + j) : 0.f,
+                              __float_as_int(r[i].z));
+                    tl = fmaxf(tl, r[i].w);
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) {
+                    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+                    const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+                    const float u2 = __shfl_xor_sync(0xffffffffu, u, off);
+                    const int32_t i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+                    tl = fmaxf(tl, __shfl_xor_sync(0xffffffffu, tl, off));
+                    combine_u(m, s, u, idx, m2, s2, u2, i2);
+                }
             }
             if (lane == 0) {
                 a.argmax[row] = idx;
                 a.pmax[row] = 1.0f / s;
                 a.ptarget[row] = (tl > -INFINITY) ? ptx::ex2((tl - m) * kLog2e) / s : 0.0f;
+                if (a.entropy)  // H = ln Z - (u ln 2) / Z, with u in log2 units
+                    a.entropy[row] = (ptx::lg2(s) - u / s) * kLn2;
                 __threadfence();  // publish this row before the CTA signals its ticket
             }
         }

@@ -73,6 +73,7 @@ struct ScoreArgs {
     int32_t n_groups, G;
     TargetSource ts;
     float4 *part;       // [N][G]
+    float *part_u;      // [N][G], entropy variant only: sum of exp(l - m) * (l - m) * log2(e) over the pair's tiles
     int32_t *status;    // cleared by CTA 0
     int32_t *tickets;   // [n_tickets], cleared here for the finish kernel
     int32_t n_tickets;
@@ -80,6 +81,8 @@ struct ScoreArgs {
 
 struct FinishArgs {
     const float4 *part;
+    const float *part_u;  // with entropy != nullptr
+    float *entropy;       // optional: H(p) = -sum_v p_v log p_v per row
     int32_t G, N, V;
     TargetSource ts;
     const int32_t *status;
@@ -99,7 +102,9 @@ void score_schedule(int32_t n_mb, int32_t n_vt, int max_units, int32_t *n_groups
 // CTA pairs of the score kernel that can be resident at once on the current device (<= 0 on error).
 int score_max_pairs();
 
-cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream);
+// entropy: also accumulate part_u (the variant used when wino_score_rows is asked for H(p)).
+cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, bool entropy,
+                         cudaStream_t stream);
 
 cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream);
 

@@ -333,5 +333,13 @@ __device__ __forceinline__ float ex2(float x)
     return y;
 }
 
+// log2(x) on the special-function unit (lg2.approx: max absolute error about 2^-22 near 1).
+__device__ __forceinline__ float lg2(float x)
+{
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 }  // namespace ptx
 }  // namespace wino

@@ -85,6 +85,8 @@ __device__ bool wait_drain(uint32_t bar, uint32_t parity)
     return true;
 }
 
+// kEntropy: also accumulate u = sum exp(l - m) * (l - m) per row (in log2 units), for H(p) = ln Z - u ln2 / Z.
+template <bool kEntropy>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW,
                  const ScoreArgs a)
@@ -276,6 +278,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             const int64_t row = (int64_t)mb * kPairM + (int)rank * kBM + q * 32 + lane;
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
             float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tl = -INFINITY;
+            float u0 = 0.f, u1 = 0.f, u2 = 0.f, u3 = 0.f;  // entropy variant
             int32_t am = 0;
             for (int vt = col; vt < a.n_vt; vt += a.G) {
                 const int32_t v0 = vt * kBN;
@@ -316,6 +319,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                                 j0 = j;
                         am = v0 + c * 32 + j0;
                         const float scale = ptx::ex2((m - cm) * kLog2e);
+                        if (kEntropy && m != -INFINITY) {  // u' = scale * (u + (m - cm) log2(e) * s)
+                            const float dl = (m - cm) * kLog2e;
+                            u0 = scale * fmaf(dl, s0, u0);
+                            u1 = scale * fmaf(dl, s1, u1);
+                            u2 = scale * fmaf(dl, s2, u2);
+                            u3 = scale * fmaf(dl, s3, u3);
+                        }
                         s0 *= scale;
                         s1 *= scale;
                         s2 *= scale;
@@ -323,12 +333,32 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         m = cm;
                     }
                     const float mb2 = m * kLog2e;
+                    if (!kEntropy) {
 #pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        s0 += ptx::ex2(fmaf(x[j + 0], kLog2e, -mb2));
-                        s1 += ptx::ex2(fmaf(x[j + 1], kLog2e, -mb2));
-                        s2 += ptx::ex2(fmaf(x[j + 2], kLog2e, -mb2));
-                        s3 += ptx::ex2(fmaf(x[j + 3], kLog2e, -mb2));
+                        for (int j = 0; j < 32; j += 4) {
+                            s0 += ptx::ex2(fmaf(x[j + 0], kLog2e, -mb2));
+                            s1 += ptx::ex2(fmaf(x[j + 1], kLog2e, -mb2));
+                            s2 += ptx::ex2(fmaf(x[j + 2], kLog2e, -mb2));
+                            s3 += ptx::ex2(fmaf(x[j + 3], kLog2e, -mb2));
+                        }
+                    } else {
+                        // t = (l - m) log2(e), kept finite (masked columns are -inf; 2^-200 is 0 in fp32 anyway)
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4) {
+                            const float t0 = fmaxf(fmaf(x[j + 0], kLog2e, -mb2), -200.f);
+                            const float t1 = fmaxf(fmaf(x[j + 1], kLog2e, -mb2), -200.f);
+                            const float t2 = fmaxf(fmaf(x[j + 2], kLog2e, -mb2), -200.f);
+                            const float t3 = fmaxf(fmaf(x[j + 3], kLog2e, -mb2), -200.f);
+                            const float e0 = ptx::ex2(t0), e1 = ptx::ex2(t1), e2 = ptx::ex2(t2), e3 = ptx::ex2(t3);
+                            s0 += e0;
+                            s1 += e1;
+                            s2 += e2;
+                            s3 += e3;
+                            u0 = fmaf(e0, t0, u0);
+                            u1 = fmaf(e1, t1, u1);
+                            u2 = fmaf(e2, t2, u2);
+                            u3 = fmaf(e3, t3, u3);
+                        }
                     }
                     const int tj = tgt - (v0 + c * 32);
                     if ((unsigned)tj < 32u) {
@@ -347,8 +377,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                     acc_phase ^= 1u;
                 }
             }
-            if (!aborted && row < a.N)
+            if (!aborted && row < a.N) {
                 a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tl);
+                if (kEntropy)
+                    a.part_u[row * a.G + col] = (u0 + u1) + (u2 + u3);
+            }
         }
     }
 
@@ -415,14 +448,16 @@ int configure_device()
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
         return -1;
     if (!done[dev]) {
-        if (cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScoreSmemBytes) !=
-            cudaSuccess)
+        if (cudaFuncSetAttribute(score_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kScoreSmemBytes) != cudaSuccess ||
+            cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kScoreSmemBytes) != cudaSuccess)
             return -1;
         cudaLaunchAttribute attr[2];
         cudaLaunchConfig_t cfg = score_config(2, nullptr, attr);
         cfg.numAttrs = 1;  // the cluster shape is what matters for the occupancy query
         int clusters = 0;
-        if (cudaOccupancyMaxActiveClusters(&clusters, score_kernel, &cfg) != cudaSuccess || clusters < 1)
+        if (cudaOccupancyMaxActiveClusters(&clusters, score_kernel<false>, &cfg) != cudaSuccess || clusters < 1)
             return -1;
         pairs[dev] = clusters;
         done[dev] = true;
@@ -434,13 +469,15 @@ int configure_device()
 
 int score_max_pairs() { return configure_device(); }
 
-cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, cudaStream_t stream)
+cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const ScoreArgs &a, bool entropy,
+                         cudaStream_t stream)
 {
     if (configure_device() < 1)
         return cudaErrorUnknown;
     cudaLaunchAttribute attr[2];
     cudaLaunchConfig_t cfg = score_config((unsigned)(2 * a.n_groups * a.G), stream, attr);
-    return cudaLaunchKernelEx(&cfg, score_kernel, tmH, tmW, a);
+    return entropy ? cudaLaunchKernelEx(&cfg, score_kernel<true>, tmH, tmW, a)
+                   : cudaLaunchKernelEx(&cfg, score_kernel<false>, tmH, tmW, a);
 }
 
 }  // namespace wino

@@ -23,10 +23,10 @@ constexpr size_t kAlign = 256;
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Workspace layout: [status | tickets[ceil(N/2)] | partial records [N][R] | argmax[N] | pmax[N] | ptarget[N]],
-// R = min(ceil(V/kBN), kMaxRecordsPerRow) bounds the records per row of any device.
+// Workspace layout: [status | tickets[ceil(N/2)] | partial records [N][R] | entropy partials [N][R] |
+// argmax[N] | pmax[N] | ptarget[N]], R = min(ceil(V/kBN), kMaxRecordsPerRow) bounds the records per row.
 struct WsLayout {
-    size_t status, tickets, part, argmax, pmax, ptarget, total;
+    size_t status, tickets, part, part_u, argmax, pmax, ptarget, total;
 };
 
 WsLayout ws_layout(int64_t N, int64_t V)
@@ -37,7 +37,8 @@ WsLayout ws_layout(int64_t N, int64_t V)
     L.status = 0;
     L.tickets = kAlign;
     L.part = L.tickets + round_up((size_t)((N + 1) / 2) * 4, kAlign);
-    L.argmax = L.part + round_up((size_t)N * (size_t)R * sizeof(float4), kAlign);
+    L.part_u = L.part + round_up((size_t)N * (size_t)R * sizeof(float4), kAlign);
+    L.argmax = L.part_u + round_up((size_t)N * (size_t)R * sizeof(float), kAlign);
     L.pmax = L.argmax + round_up((size_t)N * 4, kAlign);
     L.ptarget = L.pmax + round_up((size_t)N * 4, kAlign);
     L.total = L.ptarget + round_up((size_t)N * 4, kAlign);
@@ -190,8 +191,8 @@ int check_params(const wino_params *p)
 // Score N rows into (argmax, pmax, ptarget), and with `step` also apply Eq. 4:
 // the score kernel followed by the finish kernel.
 int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
-                     int32_t *argmax, float *pmax, float *ptarget, void *ws, size_t ws_bytes, const wino_params *step,
-                     int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream)
+                     int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws, size_t ws_bytes,
+                     const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream)
 {
     DeviceInfo info;
     int rc = device_info(&info);
@@ -219,15 +220,18 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     score_schedule(a.n_mb, a.n_vt, std::min(max_pairs, info.sm_count / 2), &a.n_groups, &a.G);
     a.ts = ts;
     a.part = reinterpret_cast<float4 *>(w8 + L.part);
+    a.part_u = reinterpret_cast<float *>(w8 + L.part_u);
     a.status = reinterpret_cast<int32_t *>(w8 + L.status);
     a.tickets = reinterpret_cast<int32_t *>(w8 + L.tickets);
     a.n_tickets = step ? step->n_seq : 0;
     prof_record(0, stream);
-    if (launch_score(tmH, tmW, a, stream) != cudaSuccess)
+    if (launch_score(tmH, tmW, a, entropy != nullptr, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
     prof_record(1, stream);
     FinishArgs f{};
     f.part = a.part;
+    f.part_u = a.part_u;
+    f.entropy = entropy;
     f.G = a.G;
     f.N = a.N;
     f.V = a.V;
@@ -283,7 +287,8 @@ int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
 }
 
 int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const int32_t *target,
-                    int32_t *argmax, float *pmax, float *ptarget, void *ws, size_t ws_bytes, void *stream)
+                    int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws, size_t ws_bytes,
+                    void *stream)
 {
     if (!H || !W || !argmax || !pmax || !ptarget || !ws)
         return WINO_ERR_ARG;
@@ -293,8 +298,8 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
         return WINO_ERR_SHAPE;
     TargetSource ts{};
     ts.target = target;
-    return score_and_finish(H, W, N, d, V, ts, argmax, pmax, ptarget, ws, ws_bytes, nullptr, nullptr, nullptr,
-                            nullptr, static_cast<cudaStream_t>(stream));
+    return score_and_finish(H, W, N, d, V, ts, argmax, pmax, ptarget, entropy, ws, ws_bytes, nullptr, nullptr,
+                            nullptr, nullptr, static_cast<cudaStream_t>(stream));
 }
 
 int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
@@ -341,7 +346,7 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     ts.blk_start = p->blk_start;
     ts.blk_len = p->blk_len;
     ts.mask_id = p->mask_id;
-    return score_and_finish(H, W, N, d, V, ts, am, pm, pt, ws, ws_bytes, p, tokens, counts, flags,
+    return score_and_finish(H, W, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags,
                             static_cast<cudaStream_t>(stream));
 }
 

@@ -42,9 +42,11 @@ class GpuStats:
     argmax: np.ndarray
     pmax: np.ndarray
     ptarget: np.ndarray
+    entropy: np.ndarray | None = None
 
 
-def gpu_score(Hd: torch.Tensor, Wd: torch.Tensor, target: np.ndarray | None, canary: int = 64) -> GpuStats:
+def gpu_score(Hd: torch.Tensor, Wd: torch.Tensor, target: np.ndarray | None, canary: int = 64,
+              entropy: bool = False) -> GpuStats:
     """wino_score_rows with guard zones after every output (checked untouched)."""
     N, d = Hd.shape
     V = Wd.shape[0]
@@ -52,13 +54,19 @@ def gpu_score(Hd: torch.Tensor, Wd: torch.Tensor, target: np.ndarray | None, can
     am = torch.full((N + canary,), -777, dtype=torch.int32, device="cuda")
     pm = torch.full((N + canary,), -7.0, dtype=torch.float32, device="cuda")
     pt = torch.full((N + canary,), -7.0, dtype=torch.float32, device="cuda")
+    en = torch.full((N + canary,), -7.0, dtype=torch.float32, device="cuda") if entropy else None
     ws = wino.workspace(N, d, V)
-    wino.wino_score_rows(Hd, Wd, t, am, pm, pt, ws, N=N, d=d, V=V)
+    wino.wino_score_rows(Hd, Wd, t, am, pm, pt, ws, entropy=en, N=N, d=d, V=V)
     torch.cuda.synchronize()
     assert wino.wino_read_device_status(ws) == wino.WINO_OK
     am, pm, pt = host(am), host(pm), host(pt)
     assert np.all(am[N:] == -777) and np.all(pm[N:] == -7.0) and np.all(pt[N:] == -7.0), "output guard zone written"
-    return GpuStats(am[:N], pm[:N], pt[:N])
+    ent = None
+    if entropy:
+        ent = host(en)
+        assert np.all(ent[N:] == -7.0), "entropy guard zone written"
+        ent = ent[:N]
+    return GpuStats(am[:N], pm[:N], pt[:N], ent)
 
 
 def compare_rows(o: oracle.RowStats, g: GpuStats, rows=None) -> dict:
@@ -70,6 +78,10 @@ def compare_rows(o: oracle.RowStats, g: GpuStats, rows=None) -> dict:
     dt = np.abs(pt.astype(np.float64) - o.ptarget)
     assert dp.max(initial=0) <= PROB_TOL, f"pmax off by {dp.max()} at row {idx[dp.argmax()]}"
     assert dt.max(initial=0) <= PROB_TOL, f"ptarget off by {dt.max()} at row {idx[dt.argmax()]}"
+    if g.entropy is not None:
+        de = np.abs(g.entropy[idx].astype(np.float64) - o.entropy)
+        assert np.all(np.isfinite(g.entropy[idx])) and de.max(initial=0) <= PROB_TOL, \
+            f"entropy off by {de.max()} at row {idx[de.argmax()]}"
     near = o.gap < TIE_TOL
     bad = (am != o.argmax) & ~near
     assert not bad.any(), f"argmax differs at rows {idx[bad][:10]}: gpu {am[bad][:10]} oracle {o.argmax[bad][:10]}"

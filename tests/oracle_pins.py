@@ -60,6 +60,7 @@ def pin_zero_hidden_is_uniform(O):
         assert r.ptarget[0] == 1.0 / V and r.ptarget[1] == 1.0 / V and r.ptarget[2] == 0.0, r.ptarget
         assert np.all(r.maxlogit == 0.0)
         assert np.allclose(r.logz, np.log(V), rtol=0, atol=1e-15)
+        assert np.allclose(r.entropy, np.log(V), rtol=1e-13, atol=1e-15)  # the uniform distribution
         if V > 1:
             assert np.all(r.gap == 0.0)
 
@@ -80,6 +81,8 @@ def pin_one_hot_weights(O):
     assert np.allclose(r.pmax, p.max(axis=1), rtol=1e-14, atol=0)
     want_t = np.array([p[n, t] if t >= 0 else 0.0 for n, t in enumerate(tgt)])
     assert np.allclose(r.ptarget, want_t, rtol=1e-14, atol=0)
+    from scipy.stats import entropy
+    assert np.allclose(r.entropy, entropy(p, axis=1), rtol=1e-12, atol=0)
 
 
 def _exact_stats(H, W, tgt):
@@ -99,7 +102,9 @@ def _exact_stats(H, W, tgt):
         t = int(tgt[n])
         pt = (mpmath.exp(mpmath.mpf((logit[t] - m).numerator) / (logit[t] - m).denominator) / Z) if 0 <= t < len(
             logit) else mpmath.mpf(0)
-        out.append((a, float(1 / Z), float(pt), gap, m))
+        ps = [mpmath.exp(mpmath.mpf((x - m).numerator) / (x - m).denominator) / Z for x in logit]
+        ent = -mpmath.fsum(q * mpmath.log(q) for q in ps if q > 0)
+        out.append((a, float(1 / Z), float(pt), gap, m, float(ent)))
     return out
 
 
@@ -114,7 +119,8 @@ def pin_exact_brute_force(O):
         tgt = rng.integers(-1, V, size=N).astype(np.int32)
         r = O.score_rows(H, W, tgt)
         ex = _exact_stats(H, W, tgt)
-        for n, (a, pm, pt, gap, m) in enumerate(ex):
+        for n, (a, pm, pt, gap, m, ent) in enumerate(ex):
+            assert abs(r.entropy[n] - ent) <= 1e-12 * max(1.0, ent), (n, r.entropy[n], ent)
             assert r.argmax[n] == a, (n, r.argmax[n], a)
             assert abs(r.pmax[n] - pm) <= 1e-13 * pm, (n, r.pmax[n], pm)
             assert abs(r.ptarget[n] - pt) <= 1e-13 * max(pt, 1e-300), (n, r.ptarget[n], pt)
@@ -137,6 +143,8 @@ def pin_library_path_rectangular(O):
     want_t = np.where(tgt >= 0, np.exp(Lg[np.arange(N), np.maximum(tgt, 0)] - lse), 0.0)
     assert np.allclose(r.ptarget, want_t, rtol=1e-12, atol=1e-300)
     assert np.allclose(r.logz, lse, rtol=1e-13, atol=0)
+    P = np.exp(Lg - lse[:, None])
+    assert np.allclose(r.entropy, -(P * np.log(P)).sum(axis=1), rtol=1e-11, atol=0)
     srt = np.sort(Lg, axis=1)
     assert np.allclose(r.gap, srt[:, -1] - srt[:, -2], rtol=0, atol=1e-12)
 

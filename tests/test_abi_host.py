@@ -59,12 +59,13 @@ def _p(**kw):
 
 def test_score_rows_argument_errors():
     L = wino.lib()
-    ok = dict(H=FAKE, W=FAKE, N=64, d=64, V=100, t=None, a=FAKE, pm=FAKE, pt=FAKE, ws=FAKE, wsb=1 << 20, s=None)
+    ok = dict(H=FAKE, W=FAKE, N=64, d=64, V=100, t=None, a=FAKE, pm=FAKE, pt=FAKE, ent=None, ws=FAKE, wsb=1 << 20,
+              s=None)
 
     def call(**kw):
         a = dict(ok, **kw)
-        return L.wino_score_rows(a["H"], a["W"], a["N"], a["d"], a["V"], a["t"], a["a"], a["pm"], a["pt"], a["ws"],
-                                 a["wsb"], a["s"])
+        return L.wino_score_rows(a["H"], a["W"], a["N"], a["d"], a["V"], a["t"], a["a"], a["pm"], a["pt"], a["ent"],
+                                 a["ws"], a["wsb"], a["s"])
     for k in ("H", "W", "a", "pm", "pt", "ws"):
         assert call(**{k: None}) == wino.WINO_ERR_ARG, k
     assert call(H=FAKE + 2) == wino.WINO_ERR_ARG

@@ -31,6 +31,9 @@ def test_score_rows_matches_oracle(N, d, V):
     o = oracle.score_rows(H, W, target)
     g = gpu_score(dev(H), dev(W), target)
     rep = compare_rows(o, g)
+    ge = gpu_score(dev(H), dev(W), target, entropy=True)  # the entropy variant of the kernel
+    compare_rows(o, ge)
+    assert np.array_equal(ge.argmax, g.argmax)
     print(f"N={N} d={d} V={V}: {rep}")
 
 
@@ -98,7 +101,7 @@ def test_score_rows_llada_shape_sampled(llada_head):
     st = ws.initial_state(w)
     H = ws.hidden_states(w, W, st, step=0)
     t = ws.row_targets_planted(w, st)
-    g = gpu_score(dev(H), Wd, t)
+    g = gpu_score(dev(H), Wd, t, entropy=True)
     rows = np.random.default_rng(0).choice(w.N, 24, replace=False)
     rows[:2] = [0, w.N - 1]
     o = oracle.score_rows(H[rows], W, t[rows])

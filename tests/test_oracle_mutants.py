@@ -42,6 +42,8 @@ MUTANTS = [
      "target[(s * 2 + 0) * blk_len + l] = (y == mask_id) ? -1 : y;"),
     ("remask_not_counted", "++remasked;", ""),
     ("left_counts_old_state", "left += (y[l] == mask_id);", "left += (prev[l] == mask_id);"),
+    ("entropy_sign_flip", "h -= p * log(p);", "h += p * log(p);"),
+    ("entropy_unnormalised", "const double p = exp(logit[v] - m) / Z;", "const double p = exp(logit[v] - m);"),
     ("freeze_ignored", "if (freeze_finished && n_mask == 0) {", "if (0) {"),
     ("freeze_always", "if (freeze_finished && n_mask == 0) {", "if (n_mask == 0) {"),
     ("last_change_on_every_position", "if (last_change && y[l] != before)", "if (last_change)"),
