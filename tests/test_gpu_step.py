@@ -341,3 +341,37 @@ def test_decode_loop_wino_plus_lockstep():
     assert not np.any(final[:, w.prompt_len:] == w.mask_id)
     assert all(b.remasked == 0 for b in stats.blocks)
     print("WINO+ loop steps/block", [b.steps for b in stats.blocks])
+
+
+@pytest.mark.parametrize("gen", [256, 512])
+def test_decode_loop_full_diffusion_lockstep(gen):
+    """Full diffusion decoding (Sec. 6.3.2): one block spanning the whole generation (256 and 512 tokens),
+    every step re-run by the oracle from the same state."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import compare_step, dev, host
+    w = ws.Workload(f"full_diffusion_{gen}", d=128, V=2000, n_seq=2, blk_len=gen, bias=((1.0, 0.0, 8.0),),
+                    n_blocks=1, bias_step=0.3, tau1=0.6, tau2=0.9)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    tok_d = dev(st.tokens)
+    rec = {}
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        H = ws.hidden_states(w, W, st, step=k)
+        rec["pre"], rec["H"] = host(tok_d).copy(), H
+        return dev(H)
+
+    reps = []
+
+    def on_step(k, b0, counts, flags):
+        o = oracle.step(rec["H"], W, rec["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2, freeze_finished=True)
+        reps.append(compare_step(rec["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1, w.tau2))
+
+    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=1, tau1=w.tau1,
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=2000)
+    final = host(tok_d)
+    assert not np.any(final[:, w.prompt_len:] == w.mask_id)
+    print(f"full diffusion gen {gen}: {stats.total_steps} steps, remasked {stats.blocks[0].remasked}, "
+          f"flagged {sum(r['flagged_positions'] for r in reps)}")
