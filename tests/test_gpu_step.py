@@ -349,8 +349,10 @@ def test_decode_loop_full_diffusion_lockstep(gen):
     every step re-run by the oracle from the same state."""
     import paper_2605_16941_gb300.loop as loop
     from gpu_helpers import compare_step, dev, host
+    # Both ends of the bias law grow: with independent per-step biases a long block only settles once
+    # every position clears verification in the same step.
     w = ws.Workload(f"full_diffusion_{gen}", d=128, V=2000, n_seq=2, blk_len=gen, bias=((1.0, 0.0, 8.0),),
-                    n_blocks=1, bias_step=0.3, tau1=0.6, tau2=0.9)
+                    n_blocks=1, bias_step=0.3, bias_floor_step=0.1, tau1=0.6, tau2=0.9)
     W = ws.weights(w)
     Wd = dev(W)
     st = ws.initial_state(w)
@@ -370,7 +372,7 @@ def test_decode_loop_full_diffusion_lockstep(gen):
         reps.append(compare_step(rec["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1, w.tau2))
 
     stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=1, tau1=w.tau1,
-                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=2000)
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=400)
     final = host(tok_d)
     assert not np.any(final[:, w.prompt_len:] == w.mask_id)
     print(f"full diffusion gen {gen}: {stats.total_steps} steps, remasked {stats.blocks[0].remasked}, "

@@ -109,6 +109,7 @@ class Workload:
     seed: int = 0
     hold: float = 0.0  # fraction of pre-decoded positions that hold their planted target
     bias_step: float = 0.0  # growth of every component's upper bound per global step
+    bias_floor_step: float = 0.0  # growth of every component's lower bound per global step
     shadow: bool = True  # False: WINO+ inference, block rows only (no verification rows)
 
     @property
@@ -201,8 +202,8 @@ def row_biases(w: Workload, step: int = 0) -> np.ndarray:
     cum = np.cumsum(wts / wts.sum())
     u = rng.random(w.N)
     comp = np.minimum(np.searchsorted(cum, u, side="right"), len(w.bias) - 1)
-    lo = np.array([c[1] for c in w.bias])[comp]
-    hi = np.array([c[2] for c in w.bias])[comp] + w.bias_step * step
+    lo = np.array([c[1] for c in w.bias])[comp] + w.bias_floor_step * step
+    hi = np.maximum(np.array([c[2] for c in w.bias])[comp] + w.bias_step * step, lo)
     return (lo + (hi - lo) * rng.random(w.N)).astype(np.float32)
 
 
