@@ -100,6 +100,17 @@ typedef struct {
 #define WINO_OPT_NO_SHADOW 2
 
 /*
+ * WINO_OPT_COMPACT (wino_step only): Eq. 4 reads, per position, only the
+ * block row of a masked position (Eq. 2) and only the shadow row of a
+ * decoded one (Eq. 3).  With this option the step first gathers that one row
+ * per position into the workspace and scores n_seq*blk_len rows instead of
+ * 2*n_seq*blk_len; the token state, counts and flags are those of the full
+ * step.  H keeps the full [s][kind][l] layout; the workspace must hold
+ * wino_workspace_size_step() bytes.
+ */
+#define WINO_OPT_COMPACT 4
+
+/*
  * Bytes of scratch the score path needs for N rows of dimension d over a
  * vocabulary of V entries (per-tile partial softmax statistics, targets and
  * per-row results, plus one status word).  `ws` passed to wino_score_rows /
@@ -108,6 +119,13 @@ typedef struct {
  * wino_score_rows.
  */
 WINO_API int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes);
+
+/*
+ * Workspace bytes wino_step needs for these parameters (row layout and
+ * WINO_OPT_COMPACT taken into account); >= wino_workspace_size of the rows it
+ * scores.
+ */
+WINO_API int wino_workspace_size_step(const wino_params *p, int64_t d, int64_t V, size_t *bytes);
 
 /*
  * Fused LM-head GEMM + full-vocabulary softmax statistics (the p_theta(.|Y~)
@@ -205,6 +223,15 @@ WINO_API int wino_read_device_status(const void *ws, void *stream, int *device_s
  */
 WINO_API int wino_profile_begin(int max_launches);
 WINO_API int wino_profile_end(double *score_ms_total, int *score_launches);
+
+/*
+ * Self-test of the failure path (device-side timeout handling; the paper has
+ * no counterpart).  Enqueues one small kernel that waits, with the library's
+ * bounded wait shortened to limit_ns (1 us .. 1 s), on a barrier nothing
+ * arrives on; it gives up, writes WINO_ERR_DEVICE_TIMEOUT to *status (device
+ * int32) and exits normally, leaving the context usable.
+ */
+WINO_API int wino_selftest_wait_timeout(int32_t *status, int64_t limit_ns, void *stream);
 
 /* Static description of a status code. */
 WINO_API const char *wino_status_string(int status);

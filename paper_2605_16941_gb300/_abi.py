@@ -29,10 +29,11 @@ FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0,
 # wino_params.options
 WINO_OPT_FREEZE_FINISHED = 1
 WINO_OPT_NO_SHADOW = 2
+WINO_OPT_COMPACT = 4
 
-EXPORTS = ("wino_workspace_size", "wino_score_rows", "wino_draft_verify", "wino_step",
+EXPORTS = ("wino_workspace_size", "wino_workspace_size_step", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
-           "wino_status_string", "wino_version")
+           "wino_selftest_wait_timeout", "wino_status_string", "wino_version")
 
 # size of the fixed device array behind wino_step_static_scratch
 WINO_STATIC_SCRATCH_BYTES = 16 << 20
@@ -65,6 +66,8 @@ def lib() -> C.CDLL:
         i64, vp, sz = C.c_int64, C.c_void_p, C.c_size_t
         L.wino_workspace_size.restype = C.c_int
         L.wino_workspace_size.argtypes = [i64, i64, i64, C.POINTER(sz)]
+        L.wino_workspace_size_step.restype = C.c_int
+        L.wino_workspace_size_step.argtypes = [C.POINTER(WinoParams), i64, i64, C.POINTER(sz)]
         L.wino_score_rows.restype = C.c_int
         L.wino_score_rows.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, vp, vp, vp, sz, vp]
         L.wino_draft_verify.restype = C.c_int
@@ -79,6 +82,8 @@ def lib() -> C.CDLL:
         L.wino_profile_begin.argtypes = [C.c_int]
         L.wino_profile_end.restype = C.c_int
         L.wino_profile_end.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_int)]
+        L.wino_selftest_wait_timeout.restype = C.c_int
+        L.wino_selftest_wait_timeout.argtypes = [vp, i64, vp]
         L.wino_status_string.restype = C.c_char_p
         L.wino_status_string.argtypes = [C.c_int]
         L.wino_version.restype = C.c_int
@@ -123,6 +128,18 @@ def wino_workspace_size(N: int, d: int, V: int) -> int:
     return out.value
 
 
+def wino_workspace_size_step(params: WinoParams, d: int, V: int) -> int:
+    out = C.c_size_t(0)
+    _check(lib().wino_workspace_size_step(C.byref(params), d, V, C.byref(out)), "wino_workspace_size_step")
+    return out.value
+
+
+def step_workspace(params: WinoParams, d: int, V: int, device=None):
+    """A zeroed uint8 device tensor of wino_workspace_size_step bytes (allocated by PyTorch)."""
+    import torch
+    return torch.zeros(wino_workspace_size_step(params, d, V), dtype=torch.uint8, device=device or "cuda")
+
+
 def workspace(N: int, d: int, V: int, device=None):
     """A zeroed uint8 device tensor of wino_workspace_size(N, d, V) bytes (allocated by PyTorch)."""
     import torch
@@ -131,8 +148,9 @@ def workspace(N: int, d: int, V: int, device=None):
 
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
                 max_steps: int = 4096, freeze_finished: bool = False, step_index: int = 0,
-                last_change=None, no_shadow: bool = False) -> WinoParams:
-    opts = (WINO_OPT_FREEZE_FINISHED if freeze_finished else 0) | (WINO_OPT_NO_SHADOW if no_shadow else 0)
+                last_change=None, no_shadow: bool = False, compact: bool = False) -> WinoParams:
+    opts = ((WINO_OPT_FREEZE_FINISHED if freeze_finished else 0) | (WINO_OPT_NO_SHADOW if no_shadow else 0) |
+            (WINO_OPT_COMPACT if compact else 0))
     return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps, opts, step_index,
                       _ptr(last_change))
 
@@ -189,3 +207,9 @@ def wino_profile_end() -> tuple[float, int]:
     ms, n = C.c_double(0), C.c_int(0)
     _check(lib().wino_profile_end(C.byref(ms), C.byref(n)), "wino_profile_end")
     return ms.value, n.value
+
+
+def wino_selftest_wait_timeout(status, limit_ns: int, stream=None) -> None:
+    """Run the bounded-wait timeout self-test; ``status`` (device int32) receives the outcome."""
+    _check(lib().wino_selftest_wait_timeout(_ptr(status), int(limit_ns), _stream(stream)),
+           "wino_selftest_wait_timeout")

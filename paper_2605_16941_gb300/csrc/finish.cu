@@ -97,9 +97,10 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
     const int L = p.blk_len;
     const int32_t mask = p.mask_id;
     const bool shadow = !(p.options & WINO_OPT_NO_SHADOW);  // WINO+ inference has no verification rows
+    const bool compact = (p.options & WINO_OPT_COMPACT) != 0;  // one row per position
     int32_t *y = tokens + (int64_t)s * p.seq_len + p.blk_start;
-    const int64_t rb = (int64_t)(shadow ? 2 * s : s) * L;  // kind-0 rows: the block Y_cur
-    const int64_t rs = (int64_t)(2 * s + 1) * L;           // kind-1 rows: the shadow block Y_shad
+    const int64_t rb = (int64_t)((shadow && !compact) ? 2 * s : s) * L;  // rows read for masked positions
+    const int64_t rs = (int64_t)(compact ? s : 2 * s + 1) * L;         // rows read for decoded positions
 
     int32_t yv[kPer], av[kPer];
     float pm[kPer], pt[kPer];
@@ -304,7 +305,8 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
     __syncthreads();
     if (threadIdx.x == 0) {
         int32_t nd = 0;
-        const int64_t per_seq = ((a.p.options & WINO_OPT_NO_SHADOW) ? 1 : 2) * (int64_t)a.p.blk_len;
+        const int64_t per_seq =
+            ((a.p.options & (WINO_OPT_NO_SHADOW | WINO_OPT_COMPACT)) ? 1 : 2) * (int64_t)a.p.blk_len;
         const int64_t rend = min(row0 + kFinishRows, (int64_t)a.N);
         for (int64_t r = row0; r < rend;) {
             const int64_t sq = r / per_seq;
@@ -332,7 +334,40 @@ __global__ void __launch_bounds__(kFinishRows * 32)
     eq4_block(blockIdx.x, tokens, argmax, pmax, ptarget, p, counts, flags, WINO_OK, sm);
 }
 
+// Row compaction: one CTA per position copies the one row Eq. 4 will read -- the block row of a masked
+// position, the shadow row of a decoded one -- with 16-byte loads (d % 8 == 0).
+__global__ void __launch_bounds__(256) gather_compact_kernel(const uint4 *__restrict__ H, uint4 *__restrict__ Hc,
+                                                             const int32_t *__restrict__ tokens, const wino_params p,
+                                                             int64_t vec_per_row)
+{
+    ptx::grid_dep_wait();  // the token state may still be being written by the previous step
+    ptx::grid_dep_launch_dependents();  // the score kernel may set up now; it waits for these rows itself
+    const int64_t r = blockIdx.x;  // = s * L + l
+    const int64_t s = r / p.blk_len, l = r - s * p.blk_len;
+    const bool masked = tokens[s * p.seq_len + p.blk_start + l] == p.mask_id;
+    const uint4 *src = H + ((2 * s + (masked ? 0 : 1)) * p.blk_len + l) * vec_per_row;
+    uint4 *dst = Hc + r * vec_per_row;
+    for (int64_t i = threadIdx.x; i < vec_per_row; i += blockDim.x)
+        dst[i] = __ldg(src + i);
+}
+
 }  // namespace
+
+cudaError_t launch_gather_compact(const uint16_t *H, uint16_t *Hc, const int32_t *tokens, const wino_params &p,
+                                  int64_t d, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((int64_t)p.n_seq * p.blk_len));
+    cfg.blockDim = dim3(256);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gather_compact_kernel, reinterpret_cast<const uint4 *>(H),
+                              reinterpret_cast<uint4 *>(Hc), tokens, p, d / 8);
+}
 
 cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream)
 {

@@ -36,6 +36,7 @@ struct TargetSource {
     const int32_t *target;  // explicit per-row targets (wino_score_rows), or nullptr
     const int32_t *tokens;  // or gathered from the token state (wino_step), or nullptr
     int32_t seq_len, blk_start, blk_len, mask_id;
+    int32_t compact;        // rows are one per position (s, l) -> row s*blk_len + l (WINO_OPT_COMPACT)
 };
 
 // Target of row `row`: explicit, or the current token of the position a
@@ -45,6 +46,11 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
     int32_t t = -1;
     if (ts.target) {
         t = ts.target[row];
+    } else if (ts.tokens && ts.compact) {
+        // one row per position: a decoded position's row is its shadow row, scored against its token
+        const int64_t s = row / ts.blk_len, l = row - s * ts.blk_len;
+        const int32_t y = ts.tokens[s * ts.seq_len + ts.blk_start + l];
+        t = (y == ts.mask_id) ? -1 : y;
     } else if (ts.tokens) {
         const int64_t two_l = 2 * (int64_t)ts.blk_len;
         const int64_t s = row / two_l, r = row - s * two_l;
@@ -77,6 +83,7 @@ struct ScoreArgs {
     int32_t *status;    // cleared by CTA 0
     int32_t *tickets;   // [n_tickets], cleared here for the finish kernel
     int32_t n_tickets;
+    int32_t h_from_prev_grid;  // H is written by the kernel launched just before (row compaction): no early loads
 };
 
 struct FinishArgs {
@@ -107,6 +114,10 @@ cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const S
                          cudaStream_t stream);
 
 cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream);
+
+// Row compaction (WINO_OPT_COMPACT): Hc[s*L + l] = H[(2s + (tokens[s, b0 + l] == MASK ? 0 : 1)) * L + l].
+cudaError_t launch_gather_compact(const uint16_t *H, uint16_t *Hc, const int32_t *tokens, const wino_params &p,
+                                  int64_t d, cudaStream_t stream);
 
 cudaError_t launch_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                                 const wino_params &p, int32_t *counts, int8_t *flags, cudaStream_t stream);

@@ -31,12 +31,11 @@
 // closing cluster barrier before TMEM is released.
 #include "internal.h"
 #include "ptx.cuh"
+#include "wait.cuh"
 
 namespace wino {
 namespace {
 
-constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait
-constexpr uint64_t kDrainLimitNs = 200000000ull;   // 0.2 s for draining after an abort
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint16_t kBothCtas = 0x3;
 
@@ -51,41 +50,6 @@ struct alignas(8) Barriers {
 };
 static_assert(sizeof(Barriers) <= 256, "barrier block must fit its reserve");
 
-// Wait for phase `parity` of `bar`; false once the wait limit passed or another
-// role of this CTA aborted.  kCluster: acquire at cluster scope (barrier arrived on by the peer CTA).
-template <bool kCluster = false>
-__device__ bool wait_bounded(uint32_t bar, uint32_t parity, int32_t *abort_flag, int32_t *status)
-{
-    auto try_wait = [&] { return kCluster ? ptx::mbar_try_wait_cluster(bar, parity) : ptx::mbar_try_wait(bar, parity); };
-    if (try_wait())
-        return true;
-    const uint64_t t0 = ptx::globaltimer_ns();
-    for (uint32_t it = 1;; ++it) {
-        if (try_wait())
-            return true;
-        if ((it & 15u) == 0) {
-            if (*reinterpret_cast<volatile int32_t *>(abort_flag))
-                return false;
-            if (ptx::globaltimer_ns() - t0 > kWaitLimitNs) {
-                atomicExch(abort_flag, 1);
-                atomicExch(status, (int32_t)WINO_ERR_DEVICE_TIMEOUT);
-                return false;
-            }
-        }
-    }
-}
-
-// Bounded wait that ignores the abort flag (used only to drain after an abort).
-__device__ bool wait_drain(uint32_t bar, uint32_t parity)
-{
-    const uint64_t t0 = ptx::globaltimer_ns();
-    while (!ptx::mbar_try_wait(bar, parity))
-        if (ptx::globaltimer_ns() - t0 > kDrainLimitNs)
-            return false;
-    return true;
-}
-
-// kEntropy: also accumulate u = sum exp(l - m) * (l - m) per row (in log2 units), for H(p) = ln Z - u ln2 / Z.
 template <bool kEntropy>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW,
@@ -141,7 +105,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
     // Programmatic launch: the TMA producer and the MMA warp only read H and W, which the grid before
     // us (the finish kernel of the previous WINO call on this stream) never writes, so they start at
-    // once.  Everything that touches what that grid reads or writes -- the token state (targets), the
+    // once (unless H itself comes from the grid before us: row compaction).  Everything that touches what that grid reads or writes -- the token state (targets), the
     // partial records, the status word and the tickets -- waits for it (grid_dep_wait) first.
     ptx::grid_dep_launch_dependents();
 
@@ -162,6 +126,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         // nothing to do: the status word reports the failed allocation check
     } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer (both CTAs)
+        if (a.h_from_prev_grid)  // H was written by the grid before us (row compaction)
+            ptx::grid_dep_wait();
         const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every vocabulary tile
         const uint64_t pol_w = ptx::policy_evict_normal();  // W is shared by the row-block groups
         int stage = 0;

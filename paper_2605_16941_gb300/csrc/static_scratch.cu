@@ -50,8 +50,7 @@ extern "C" int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, in
     if (!p)
         return WINO_ERR_ARG;
     size_t need = 0;
-    const int rows_per_pos = (p->options & WINO_OPT_NO_SHADOW) ? 1 : 2;
-    const int rc = wino_workspace_size((int64_t)p->n_seq * rows_per_pos * p->blk_len, d, V, &need);
+    const int rc = wino_workspace_size_step(p, d, V, &need);
     if (rc != WINO_OK)
         return rc;
     if (need > WINO_STATIC_SCRATCH_BYTES)

@@ -192,7 +192,8 @@ int check_params(const wino_params *p)
 // the score kernel followed by the finish kernel.
 int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
                      int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws, size_t ws_bytes,
-                     const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream)
+                     const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream,
+                     bool h_from_prev_grid = false)
 {
     DeviceInfo info;
     int rc = device_info(&info);
@@ -224,6 +225,7 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     a.status = reinterpret_cast<int32_t *>(w8 + L.status);
     a.tickets = reinterpret_cast<int32_t *>(w8 + L.tickets);
     a.n_tickets = step ? step->n_seq : 0;
+    a.h_from_prev_grid = h_from_prev_grid ? 1 : 0;
     prof_record(0, stream);
     if (launch_score(tmH, tmW, a, entropy != nullptr, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
@@ -250,6 +252,22 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     if (launch_finish(f, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
     return WINO_OK;
+}
+
+// Rows wino_step scores for these parameters, and the workspace it needs.
+int64_t step_rows(const wino_params &p)
+{
+    const bool one_row = (p.options & (WINO_OPT_NO_SHADOW | WINO_OPT_COMPACT)) != 0;
+    return (int64_t)p.n_seq * (one_row ? 1 : 2) * p.blk_len;
+}
+
+size_t step_ws_bytes(const wino_params &p, int64_t d, int64_t V)
+{
+    const int64_t rows = step_rows(p);
+    size_t total = ws_layout(rows, V).total;
+    if (p.options & WINO_OPT_COMPACT)
+        total += round_up((size_t)rows * (size_t)d * 2, kAlign);  // the gathered rows
+    return total;
 }
 
 }  // namespace
@@ -283,6 +301,16 @@ int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
     if (!shape_ok(N, d, V))
         return WINO_ERR_SHAPE;
     *bytes = ws_layout(N, V).total;
+    return WINO_OK;
+}
+
+int wino_workspace_size_step(const wino_params *p, int64_t d, int64_t V, size_t *bytes)
+{
+    if (!p || !bytes)
+        return WINO_ERR_ARG;
+    if (!shape_ok(step_rows(*p), d, V))
+        return WINO_ERR_SHAPE;
+    *bytes = step_ws_bytes(*p, d, V);
     return WINO_OK;
 }
 
@@ -330,11 +358,14 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     if (rc != WINO_OK)
         return rc;
     const bool shadow = !(p->options & WINO_OPT_NO_SHADOW);
-    const int64_t N = (int64_t)p->n_seq * (shadow ? 2 : 1) * p->blk_len;
+    const bool compact = (p->options & WINO_OPT_COMPACT) != 0;
+    if (compact && !shadow)
+        return WINO_ERR_ARG;  // without a shadow block there is nothing to compact
+    const int64_t N = step_rows(*p);  // rows scored
     if (!shape_ok(N, d, V) || p->mask_id >= V)
         return WINO_ERR_SHAPE;
     const WsLayout L = ws_layout(N, V);
-    if (ws_bytes < L.total)
+    if (ws_bytes < step_ws_bytes(*p, d, V))
         return WINO_ERR_WORKSPACE;
     uint8_t *w8 = static_cast<uint8_t *>(ws);
     int32_t *am = reinterpret_cast<int32_t *>(w8 + L.argmax);
@@ -346,8 +377,20 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     ts.blk_start = p->blk_start;
     ts.blk_len = p->blk_len;
     ts.mask_id = p->mask_id;
-    return score_and_finish(H, W, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags,
-                            static_cast<cudaStream_t>(stream));
+    ts.compact = compact ? 1 : 0;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const uint16_t *Hs = H;
+    if (compact) {  // gather the one row per position Eq. 4 reads, behind the workspace proper
+        DeviceInfo info;
+        if ((rc = device_info(&info)) != WINO_OK)
+            return rc;
+        uint16_t *Hc = reinterpret_cast<uint16_t *>(w8 + L.total);
+        if (launch_gather_compact(H, Hc, tokens, *p, d, s) != cudaSuccess)
+            return WINO_ERR_CUDA;
+        Hs = Hc;
+    }
+    return score_and_finish(Hs, W, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s,
+                            compact);
 }
 
 int wino_profile_begin(int max_launches)

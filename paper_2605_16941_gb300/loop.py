@@ -15,7 +15,7 @@ from __future__ import annotations
 from dataclasses import dataclass, field
 from typing import Callable
 
-from ._abi import WINO_ERR_MAX_STEPS, WinoError, make_params, wino_step, wino_workspace_size
+from ._abi import WINO_ERR_MAX_STEPS, WinoError, make_params, wino_step, wino_workspace_size_step
 
 
 @dataclass
@@ -37,7 +37,8 @@ class LoopStats:
 
 def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float, mask_id: int,
            hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
-           on_step: Callable | None = None, last_change=None, no_shadow: bool = False) -> LoopStats:
+           on_step: Callable | None = None, last_change=None, no_shadow: bool = False,
+           compact: bool = False) -> LoopStats:
     """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
 
     ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
@@ -47,15 +48,17 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     receives, per position, the last step that changed it: after the decode, each
     position's WINO finalization step t_l (Sec. 5.1).  ``no_shadow``: WINO+ inference
     (Sec. 5.3): ``hidden`` returns only the n_seq*blk_len block rows, drafting uses the
-    single threshold ``tau1`` and nothing is re-masked.
+    single threshold ``tau1`` and nothing is re-masked.  ``compact``: score only the row
+    each position's update reads (WINO_OPT_COMPACT), same results.
     """
     import torch
 
     n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
     d, V = int(W.shape[1]), int(W.shape[0])
-    N = n_seq * (1 if no_shadow else 2) * blk_len
+    N = n_seq * (1 if (no_shadow or compact) else 2) * blk_len  # rows scored per step
     dev = tokens.device
-    ws = torch.zeros(wino_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
+    p0 = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact)
+    ws = torch.zeros(wino_workspace_size_step(p0, d, V), dtype=torch.uint8, device=dev)
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
     counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
@@ -64,7 +67,7 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     for b in range(n_blocks):
         b0 = prompt_len + b * blk_len
         p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True,
-                        last_change=last_change, no_shadow=no_shadow)
+                        last_change=last_change, no_shadow=no_shadow, compact=compact)
         bs = BlockStats(block=b, blk_start=b0)
         while True:
             if bs.steps >= max_steps:

@@ -1,0 +1,35 @@
+"""Failure detection on the GPU without faulting or hanging it: a bounded device wait that
+nothing satisfies gives up, reports WINO_ERR_DEVICE_TIMEOUT, and the context stays usable."""
+import time
+
+import numpy as np
+import pytest
+import torch
+
+import wino_synth as ws
+
+pytestmark = pytest.mark.gpu
+
+
+def test_bounded_wait_times_out_and_context_survives():
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, host
+    status = torch.full((1,), 12345, dtype=torch.int32, device="cuda")
+    t0 = time.time()
+    wino.wino_selftest_wait_timeout(status, 20_000_000)  # 20 ms
+    torch.cuda.synchronize()
+    dt = time.time() - t0
+    assert int(status.item()) == wino.WINO_ERR_DEVICE_TIMEOUT
+    assert 0.015 < dt < 5.0, dt
+    # the context still works: a normal step runs and reports OK
+    w = ws.WORKLOADS["tiny"]
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    tok = dev(st.tokens)
+    counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device="cuda")
+    wsp = wino.workspace(w.N, w.d, w.V)
+    p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len)
+    wino.wino_step(dev(ws.hidden_states(w, W, st)), dev(W), tok, p, counts, wsp)
+    torch.cuda.synchronize()
+    assert wino.wino_read_device_status(wsp) == wino.WINO_OK
+    assert np.all(host(counts) >= 0)

@@ -377,3 +377,68 @@ def test_decode_loop_full_diffusion_lockstep(gen):
     assert not np.any(final[:, w.prompt_len:] == w.mask_id)
     print(f"full diffusion gen {gen}: {stats.total_steps} steps, remasked {stats.blocks[0].remasked}, "
           f"flagged {sum(r['flagged_positions'] for r in reps)}")
+
+
+def _gpu_step_opts(w, Wd, tokens, H, blk_start, compact):
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, host
+    tok_d = dev(tokens)
+    counts = torch.full((w.n_seq, 3), -9, dtype=torch.int32, device="cuda")
+    flags = torch.full((w.n_seq, w.blk_len), -9, dtype=torch.int8, device="cuda")
+    p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, blk_start, w.blk_len, compact=compact)
+    wsp = wino.step_workspace(p, w.d, w.V)
+    wino.wino_step(dev(H), Wd, tok_d, p, counts, wsp, flags=flags)
+    torch.cuda.synchronize()
+    assert wino.wino_read_device_status(wsp) == wino.WINO_OK
+    return host(tok_d), host(counts), host(flags)
+
+
+@pytest.mark.parametrize("name", ["tiny_cov", "mid_cov", "llada_b1_cov"])
+def test_step_compact_matches_full_step_and_oracle(name):
+    """Row compaction scores only the row each position's update reads; the step's result is the same."""
+    from gpu_helpers import compare_step, dev
+    base = {"tiny_cov": ws.WORKLOADS["tiny"],
+            "mid_cov": ws.Workload("mid", d=256, V=5000, n_seq=4, blk_len=64, bias=((1.0, 0.0, 10.0),),
+                                   predecoded=0.5),
+            "llada_b1_cov": ws.WORKLOADS["llada_b1"]}[name]
+    w = ws.coverage_variant(base)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    for step in range(2 if name != "llada_b1_cov" else 1):
+        H = ws.hidden_states(w, W, st, step=step)
+        tf, cf, ff = _gpu_step_opts(w, Wd, st.tokens, H, st.blk_start, compact=False)
+        tc, cc, fc = _gpu_step_opts(w, Wd, st.tokens, H, st.blk_start, compact=True)
+        o = oracle.step(H, W, st.tokens, st.blk_start, w.blk_len, w.mask_id, w.tau1, w.tau2)
+        rep = compare_step(st.tokens, tc, cc, o, st.blk_start, w.blk_len, w.mask_id, w.tau1, w.tau2)
+        if rep["flagged_positions"] == 0:
+            assert np.array_equal(tc, tf) and np.array_equal(cc, cf) and np.array_equal(fc, ff)
+        print(f"compact {name} step {step}: {rep}")
+
+
+def test_decode_loop_compact_lockstep():
+    """A decode loop with row compaction, every step re-run by the (full) oracle step."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import compare_step, dev, host
+    w = ws.Workload("compact_loop", d=64, V=1000, n_seq=2, blk_len=32, bias=((1.0, 0.0, 6.0),), n_blocks=3,
+                    bias_step=0.5, tau1=0.7, tau2=0.9)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    tok_d = dev(st.tokens)
+    rec = {}
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        H = ws.hidden_states(w, W, st, step=k)
+        rec["pre"], rec["H"] = host(tok_d).copy(), H
+        return dev(H)
+
+    def on_step(k, b0, counts, flags):
+        o = oracle.step(rec["H"], W, rec["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2, freeze_finished=True)
+        compare_step(rec["pre"], host(tok_d), counts, o, b0, w.blk_len, w.mask_id, w.tau1, w.tau2)
+
+    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=500, compact=True)
+    assert not np.any(host(tok_d)[:, w.prompt_len:] == w.mask_id)
+    assert stats.rows_scored == stats.total_steps * w.n_seq * w.blk_len
