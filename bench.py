@@ -65,7 +65,7 @@ def config_dict(w):
 class ClockSampler:
     """nvidia-smi sampling of SM clock, power and throttle reasons while the timed region runs."""
 
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw.instant,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
 
@@ -308,35 +308,72 @@ def run_wino(args, rank, world, local_rank):
         raise RuntimeError("device status not OK after the timed region")
     t_max = 1e3 * job_time_max(elapsed_ms / 1e3, world, device=dev)
 
-    # ---- end to end through the C ABI with host buffers (pinned), one host read of the result per step
+    # ---- end to end through the C ABI with host buffers (pinned): every step uploads its hidden states and
+    # token state, and the host reads that step's result (token state and counts) back.  Two buffer sets
+    # and three streams (upload, compute, download) let step i+1's upload and step i-1's download run
+    # under step i's kernels; the host reads a step's result before its buffers are reused.
     Hh = [torch.from_numpy(np.ascontiguousarray(h).view(np.int16)).pin_memory() for h in Hs]
     tok_h = torch.from_numpy(st.tokens).pin_memory()
-    tok_out = torch.empty_like(tok_h).pin_memory()
-    cnt_out = torch.empty((w.n_seq, 3), dtype=torch.int32).pin_memory()
-    Hbuf = torch.empty_like(Hd[0])
+    up, down = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    Hbuf = [torch.empty_like(Hd[0]) for _ in range(2)]
+    tokb = [torch.empty_like(tok) for _ in range(2)]
+    cntb = [torch.zeros_like(counts) for _ in range(2)]
+    tok_out = [torch.empty_like(tok_h).pin_memory() for _ in range(2)]
+    cnt_out = [torch.empty((w.n_seq, 3), dtype=torch.int32).pin_memory() for _ in range(2)]
+    ev_up = [torch.cuda.Event() for _ in range(2)]
+    ev_step = [torch.cuda.Event() for _ in range(2)]
+    ev_down = [torch.cuda.Event() for _ in range(2)]
+    pending = [False, False]
+    e2e_bad = [0]
     e2e_steps = args.steps
 
+    def consume(j):  # the host reads a finished step's result
+        ev_down[j].synchronize()
+        if int(cnt_out[j].min()) < 0 or int(tok_out[j][0, 0]) < 0:
+            e2e_bad[0] += 1
+        pending[j] = False
+
     def e2e_step(i):
-        Hbuf.copy_(Hh[i % n_h], non_blocking=True)
-        tok.copy_(tok_h, non_blocking=True)
-        wino.wino_step(Hbuf, Wd, tok, p, counts, wsp, stream=sid)
-        tok_out.copy_(tok, non_blocking=True)
-        cnt_out.copy_(counts, non_blocking=True)
-        stream.synchronize()
+        j = i % 2
+        if pending[j]:
+            consume(j)
+        with torch.cuda.stream(up):
+            up.wait_event(ev_step[j])  # step i-2 is done with these buffers
+            Hbuf[j].copy_(Hh[i % n_h], non_blocking=True)
+            tokb[j].copy_(tok_h, non_blocking=True)
+            ev_up[j].record(up)
+        stream.wait_event(ev_up[j])
+        wino.wino_step(Hbuf[j], Wd, tokb[j], p, cntb[j], wsp, stream=sid)
+        ev_step[j].record(stream)
+        with torch.cuda.stream(down):
+            down.wait_event(ev_step[j])
+            tok_out[j].copy_(tokb[j], non_blocking=True)
+            cnt_out[j].copy_(cntb[j], non_blocking=True)
+            ev_down[j].record(down)
+        pending[j] = True
+
+    def e2e_drain():
+        for j in range(2):
+            if pending[j]:
+                consume(j)
 
     for i in range(max(3, args.warmup)):
         e2e_step(i)
+    e2e_drain()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
     te0 = time.perf_counter()
     for i in range(e2e_steps):
         e2e_step(i)
+    e2e_drain()
     torch.cuda.synchronize(dev)
     te = time.perf_counter() - te0
     te = job_time_max(te, world, device=dev)
+    if e2e_bad[0]:
+        raise RuntimeError(f"{e2e_bad[0]} end-to-end steps returned an error status")
     h2d = Hh[0].numel() * 2 + tok_h.numel() * 4
-    d2h = tok_out.numel() * 4 + cnt_out.numel() * 4
+    d2h = tok_out[0].numel() * 4 + cnt_out[0].numel() * 4
 
     if rank != 0:
         if world > 1:

@@ -78,6 +78,13 @@ typedef struct {
                              decode with step_index = 1, 2, ..., it ends as each position's WINO
                              finalization step t_l = min{t : y_l^(j) = y_l^final for all j >= t}
                              (Sec. 5.1; 0 for the prompt).  NULL: not recorded. */
+    int32_t draft_m;   /* 0: drafting by Eq. 2 (tau1 plus the at-least-one rule).  M > 0: naive
+                          parallel sampling, the fixed-step-size decoding WINO is compared with
+                          (Sec. 3, Sec. 6.3.3): the min(M, #MASK) masked positions with the largest
+                          max_v p are drafted (smallest position first on equal confidence) and
+                          tau1 is not used; M = 1 is high-confidence greedy decoding (Eq. 1).
+                          Verification is unchanged; combine with WINO_OPT_NO_SHADOW for the
+                          irreversible baseline decoders.  Must be >= 0. */
 } wino_params;
 
 /*
@@ -160,9 +167,10 @@ WINO_API int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, in
  *   flags  [n_seq, blk_len] int8 out or NULL: per position 0 unchanged,
  *          1 drafted (pmax > tau1), 2 drafted by the at-least-one rule,
  *          3 re-masked, 4 selected for drafting but its argmax is MASK itself
- *          (the position stays MASK and is not counted as drafted)
+ *          (the position stays MASK and is not counted as drafted),
+ *          5 drafted by the fixed-M rule (draft_m > 0)
  * Ties in the at-least-one rule go to the smallest position.  Requires
- * 0 <= tau1, tau2 <= 1, 1 <= blk_len <= 1024, n_seq >= 1.
+ * 0 <= tau1, tau2 <= 1, 1 <= blk_len <= 1024, n_seq >= 1, draft_m >= 0.
  */
 WINO_API int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream);

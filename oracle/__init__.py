@@ -17,7 +17,7 @@ import numpy as np
 
 from .build import build as _build
 
-FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0, 1, 2, 3, 4
+FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK, FLAG_DRAFT_TOP_M = 0, 1, 2, 3, 4, 5
 
 
 def _p(a):
@@ -74,10 +74,10 @@ class Oracle:
         L.oracle_row_targets.argtypes = [vp, i64, i64, i64, i64, i32, vp]
         L.oracle_draft_verify.restype = C.c_int
         L.oracle_draft_verify.argtypes = [vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp, C.c_int,
-                                          C.c_int, i32, vp]
+                                          C.c_int, i32, vp, i64]
         L.oracle_step.restype = C.c_int
         L.oracle_step.argtypes = [vp, vp, i64, i64, vp, i64, i64, i64, i64, i32, dbl, dbl, vp, vp, vp, vp, vp,
-                                  vp, C.c_int, C.c_int, C.c_int, i32, vp]
+                                  vp, C.c_int, C.c_int, C.c_int, i32, vp, i64]
         L.oracle_num_threads.restype = C.c_int
         L.oracle_num_threads.argtypes = []
         self.L = L
@@ -126,10 +126,12 @@ class Oracle:
     def draft_verify(self, tokens: np.ndarray, blk_start: int, blk_len: int, mask_id: int, tau1: float,
                      tau2: float, argmax: np.ndarray, pmax: np.ndarray, ptarget: np.ndarray,
                      freeze_finished: bool = False, step_index: int = 0, last_change: np.ndarray | None = None,
-                     no_shadow: bool = False):
+                     no_shadow: bool = False, draft_m: int = 0):
         """Eq. 4 on a copy of ``tokens``; returns (new_tokens, counts [n_seq,3], flags [n_seq, blk_len]).
         ``last_change`` (int32 [n_seq, seq_len], updated in place) gets ``step_index`` where a token changes.
-        ``no_shadow``: WINO+ inference, rows are block rows only and ``ptarget`` may be None."""
+        ``no_shadow``: WINO+ inference, rows are block rows only and ``ptarget`` may be None.
+        ``draft_m`` > 0: draft the ``draft_m`` most confident masked positions instead (naive parallel
+        sampling, Sec. 3; 1 = greedy, Eq. 1)."""
         tok = np.array(tokens, dtype=np.int32, copy=True, order="C")
         n_seq, S = tok.shape
         N = n_seq * (1 if no_shadow else 2) * blk_len
@@ -141,15 +143,17 @@ class Oracle:
         rc = self.L.oracle_draft_verify(_p(tok), n_seq, S, blk_start, blk_len, mask_id, float(tau1),
                                         float(tau2), _p(am), _p(pm), _p(pt), _p(counts), _p(flags),
                                         int(bool(freeze_finished)), int(bool(no_shadow)), int(step_index),
-                                        _p(_lc(last_change, tok)))
+                                        _p(_lc(last_change, tok)), int(draft_m))
         if rc != 0:
             raise RuntimeError(f"oracle_draft_verify failed: {rc}")
         return tok, counts, flags
 
     def step(self, H_bits: np.ndarray, W_bits: np.ndarray, tokens: np.ndarray, blk_start: int, blk_len: int,
              mask_id: int, tau1: float, tau2: float, nthreads: int = 0, freeze_finished: bool = False,
-             step_index: int = 0, last_change: np.ndarray | None = None, no_shadow: bool = False) -> StepResult:
-        """One whole WINO step on a copy of ``tokens`` (``last_change``, ``no_shadow`` as in draft_verify)."""
+             step_index: int = 0, last_change: np.ndarray | None = None, no_shadow: bool = False,
+             draft_m: int = 0) -> StepResult:
+        """One whole WINO step on a copy of ``tokens`` (``last_change``, ``no_shadow``, ``draft_m`` as in
+        draft_verify)."""
         H, W = _c(H_bits, np.uint16), _c(W_bits, np.uint16)
         tok = np.array(tokens, dtype=np.int32, copy=True, order="C")
         n_seq, S = tok.shape
@@ -162,7 +166,7 @@ class Oracle:
         rc = self.L.oracle_step(_p(H), _p(W), d, V, _p(tok), n_seq, S, blk_start, blk_len, mask_id, float(tau1),
                                 float(tau2), _p(r.counts), _p(r.flags), _p(r.argmax), _p(r.pmax), _p(r.ptarget),
                                 _p(r.gap), nthreads, int(bool(freeze_finished)), int(bool(no_shadow)),
-                                int(step_index), _p(_lc(last_change, tok)))
+                                int(step_index), _p(_lc(last_change, tok)), int(draft_m))
         if rc != 0:
             raise RuntimeError(f"oracle_step failed: {rc}")
         return r
@@ -199,12 +203,13 @@ def row_targets(tokens, blk_start: int, blk_len: int, mask_id: int):
 
 
 def draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget, freeze_finished=False,
-                 step_index=0, last_change=None, no_shadow=False):
+                 step_index=0, last_change=None, no_shadow=False, draft_m=0):
     return default().draft_verify(tokens, blk_start, blk_len, mask_id, tau1, tau2, argmax, pmax, ptarget,
-                                  freeze_finished, step_index, last_change, no_shadow)
+                                  freeze_finished, step_index, last_change, no_shadow, draft_m)
 
 
 def step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads: int = 0,
-         freeze_finished: bool = False, step_index: int = 0, last_change=None, no_shadow: bool = False) -> StepResult:
+         freeze_finished: bool = False, step_index: int = 0, last_change=None, no_shadow: bool = False,
+         draft_m: int = 0) -> StepResult:
     return default().step(H_bits, W_bits, tokens, blk_start, blk_len, mask_id, tau1, tau2, nthreads, freeze_finished,
-                          step_index, last_change, no_shadow)
+                          step_index, last_change, no_shadow, draft_m)

@@ -173,6 +173,7 @@ int oracle_row_targets(const int32_t *tokens, int64_t n_seq, int64_t seq_len, in
 #define ORACLE_FLAG_DRAFT_FALLBACK 2 /* drafted by the at-least-one rule (Eq. 1)     */
 #define ORACLE_FLAG_REMASK 3         /* re-masked: p(current token) < tau2 (Eq. 3)   */
 #define ORACLE_FLAG_DRAFT_IS_MASK 4  /* selected for drafting but argmax is MASK     */
+#define ORACLE_FLAG_DRAFT_TOP_M 5    /* drafted by the fixed-M rule (Sec. 3)         */
 
 /*
  * One WINO step, Eq. 4, on every sequence's current block [blk_start,
@@ -195,12 +196,18 @@ int oracle_row_targets(const int32_t *tokens, int64_t n_seq, int64_t seq_len, in
  * shadow block, the rows are the block rows only ([s][l], row s*blk_len + l),
  * drafting uses the single threshold tau1 with the same at-least-one rule,
  * and R is empty (ptarget may be NULL).
+ *
+ * draft_m > 0 replaces the drafting rule by naive parallel sampling (Sec. 3,
+ * the fixed number of tokens per step of Sec. 6.3.3): D is the min(M, #MASK)
+ * masked positions with the largest pmax(block row l), the smallest l first
+ * among equal pmax; tau1 is not used.  M = 1 is high-confidence greedy
+ * decoding (Eq. 1).  Verification is unchanged (off with no_shadow).
  */
 int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t blk_start,
                         int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                         const int32_t *argmax, const double *pmax, const double *ptarget,
                         int32_t *counts, int8_t *flags, int freeze_finished, int no_shadow, int32_t step_index,
-                        int32_t *last_change)
+                        int32_t *last_change, int64_t draft_m)
 {
     if (!tokens || !argmax || !pmax || (!ptarget && !no_shadow) || !counts || n_seq < 0 || blk_len < 1 ||
         blk_start < 0 || blk_start + blk_len > seq_len)
@@ -221,7 +228,7 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
         int64_t n_draft = 0, n_mask = 0;
         for (int64_t l = 0; l < blk_len; ++l) {
             prev[l] = y[l];
-            inD[l] = (prev[l] == mask_id) && (pmax[row_blk + l] > tau1);
+            inD[l] = (draft_m <= 0) && (prev[l] == mask_id) && (pmax[row_blk + l] > tau1);
             inR[l] = !no_shadow && (prev[l] != mask_id) && (ptarget[row_shd + l] < tau2);
             n_draft += inD[l];
             n_mask += (prev[l] == mask_id);
@@ -234,7 +241,16 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
             continue;
         }
         int64_t fallback = -1;
-        if (n_draft == 0 && n_mask > 0) {
+        if (draft_m > 0) {
+            /* the M most confident masked positions: M times, take the best one not yet taken */
+            for (int64_t j = 0; j < draft_m && j < n_mask; ++j) {
+                int64_t pick = -1;
+                for (int64_t l = 0; l < blk_len; ++l)
+                    if (prev[l] == mask_id && !inD[l] && (pick < 0 || pmax[row_blk + l] > pmax[row_blk + pick]))
+                        pick = l;
+                inD[pick] = 1;
+            }
+        } else if (n_draft == 0 && n_mask > 0) {
             double best = -INFINITY;
             for (int64_t l = 0; l < blk_len; ++l)
                 if (prev[l] == mask_id && (fallback < 0 || pmax[row_blk + l] > best)) {
@@ -252,7 +268,8 @@ int oracle_draft_verify(int32_t *tokens, int64_t n_seq, int64_t seq_len, int64_t
                 if (y[l] == mask_id)
                     code = ORACLE_FLAG_DRAFT_IS_MASK;
                 else {
-                    code = (l == fallback) ? ORACLE_FLAG_DRAFT_FALLBACK : ORACLE_FLAG_DRAFT;
+                    code = (draft_m > 0) ? ORACLE_FLAG_DRAFT_TOP_M
+                                         : (l == fallback) ? ORACLE_FLAG_DRAFT_FALLBACK : ORACLE_FLAG_DRAFT;
                     ++drafted;
                 }
             } else if (inR[l]) {
@@ -286,7 +303,7 @@ int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int3
                 int64_t seq_len, int64_t blk_start, int64_t blk_len, int32_t mask_id, double tau1, double tau2,
                 int32_t *counts, int8_t *flags, int32_t *argmax_out, double *pmax_out, double *ptarget_out,
                 double *gap_out, int nthreads, int freeze_finished, int no_shadow, int32_t step_index,
-                int32_t *last_change)
+                int32_t *last_change, int64_t draft_m)
 {
     const int64_t N = n_seq * (no_shadow ? 1 : 2) * blk_len;
     int32_t *target = (int32_t *)malloc((size_t)N * sizeof(int32_t));
@@ -307,7 +324,8 @@ int oracle_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int3
             rc = oracle_score_rows(H, W, N, d, V, target, am, pm, pt, gp, NULL, NULL, NULL, nthreads);
         if (rc == ORACLE_OK)
             rc = oracle_draft_verify(tokens, n_seq, seq_len, blk_start, blk_len, mask_id, tau1, tau2, am, pm,
-                                     pt, counts, flags, freeze_finished, no_shadow, step_index, last_change);
+                                     pt, counts, flags, freeze_finished, no_shadow, step_index, last_change,
+                                     draft_m);
         if (rc == ORACLE_OK) {
             if (argmax_out)
                 memcpy(argmax_out, am, (size_t)N * sizeof(int32_t));

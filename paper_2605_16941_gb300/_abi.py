@@ -49,7 +49,7 @@ class WinoParams(C.Structure):
     _fields_ = [("tau1", C.c_float), ("tau2", C.c_float), ("mask_id", C.c_int32), ("n_seq", C.c_int32),
                 ("seq_len", C.c_int32), ("blk_start", C.c_int32), ("blk_len", C.c_int32),
                 ("max_steps", C.c_int32), ("options", C.c_int32), ("step_index", C.c_int32),
-                ("last_change", C.c_void_p)]
+                ("last_change", C.c_void_p), ("draft_m", C.c_int32)]
 
 
 def library_path() -> Path:
@@ -148,11 +148,12 @@ def workspace(N: int, d: int, V: int, device=None):
 
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
                 max_steps: int = 4096, freeze_finished: bool = False, step_index: int = 0,
-                last_change=None, no_shadow: bool = False, compact: bool = False) -> WinoParams:
+                last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0) -> WinoParams:
+    """wino_params; ``draft_m`` > 0 selects fixed-M drafting (naive parallel sampling, Sec. 3)."""
     opts = ((WINO_OPT_FREEZE_FINISHED if freeze_finished else 0) | (WINO_OPT_NO_SHADOW if no_shadow else 0) |
             (WINO_OPT_COMPACT if compact else 0))
     return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps, opts, step_index,
-                      _ptr(last_change))
+                      _ptr(last_change), draft_m)
 
 
 def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, entropy=None, N: int | None = None,

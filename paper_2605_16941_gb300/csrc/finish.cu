@@ -25,7 +25,10 @@
 // and, if no masked position clears tau1 while the block still has a MASK,
 // the masked position with the largest pmax (smallest position on ties) is
 // drafted: the greedy rule of Eq. 1, which keeps at least one token coming per
-// step.  The rules touch disjoint positions (MASK vs not MASK), so the update
+// step.  With draft_m > 0 the drafting rule is naive parallel sampling
+// instead (Sec. 3): the draft_m masked positions with the largest pmax
+// (smallest position first on ties) are drafted, whatever tau1 says.  The
+// rules touch disjoint positions (MASK vs not MASK), so the update
 // is applied in place in one pass after a CTA-wide reduction.  With
 // WINO_OPT_FREEZE_FINISHED a sequence whose block already has no MASK is left
 // as it is (its own loop, Sec. 4.2.3, has ended).
@@ -78,6 +81,7 @@ __device__ __forceinline__ void combine_u(float &m, float &s, float &u, int32_t 
 struct Eq4Smem {
     int32_t i0[kFinishRows], i1[kFinishRows], i2[kFinishRows];
     float f0[kFinishRows];
+    float conf[kMaxBlkLen];  // fixed-M drafting: pmax of each masked position, -inf elsewhere
 };
 
 // Eq. 4 on sequence s by the whole CTA (kFinishRows warps; thread t owns positions t, t + 256, ...).
@@ -169,7 +173,36 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
             counts[s * 3 + tid] = 0;
         return;
     }
-    const int fallback = (n_clear == 0 && n_mask > 0) ? best_l : -1;
+    const int fallback = (p.draft_m <= 0 && n_clear == 0 && n_mask > 0) ? best_l : -1;
+
+    // Fixed-M drafting: position l is drafted iff fewer than M masked positions rank before it
+    // (larger pmax, or equal pmax and a smaller position).
+    bool top[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i)
+        top[i] = false;
+    if (p.draft_m > 0) {
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+            const int l = tid + i * kT;
+            if (l < L)
+                sm.conf[l] = (yv[i] == mask) ? pm[i] : -INFINITY;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+            const int l = tid + i * kT;
+            if (l < L && yv[i] == mask) {
+                int before = 0;
+                for (int j = 0; j < L && before < p.draft_m; ++j) {
+                    const float c = sm.conf[j];
+                    before += (c > pm[i]) || (c == pm[i] && j < l);
+                }
+                top[i] = before < p.draft_m;
+            }
+        }
+        __syncthreads();  // conf is scratch of this sequence only
+    }
 
     // Pass 2: apply Eq. 4 simultaneously.
     int drafted = 0, remasked = 0, left = 0;
@@ -182,9 +215,9 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
         int32_t next = prev;
         int8_t code = 0;
         if (prev == mask) {
-            if (pm[i] > p.tau1 || l == fallback) {
+            if (p.draft_m > 0 ? top[i] : (pm[i] > p.tau1 || l == fallback)) {
                 next = av[i];
-                code = (next == mask) ? 4 : (l == fallback ? 2 : 1);
+                code = (next == mask) ? 4 : (p.draft_m > 0 ? 5 : (l == fallback ? 2 : 1));
             }
         } else if (shadow && pt[i] < p.tau2) {
             next = mask;
@@ -195,7 +228,7 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
             if (p.last_change)  // WINO finalization step bookkeeping (Sec. 5.1)
                 p.last_change[(int64_t)s * p.seq_len + p.blk_start + l] = p.step_index;
         }
-        drafted += (code == 1 || code == 2);
+        drafted += (code == 1 || code == 2 || code == 5);
         remasked += (code == 3);
         left += (next == mask);
         if (flags)

@@ -178,7 +178,7 @@ int check_params(const wino_params *p)
 {
     if (!p)
         return WINO_ERR_ARG;
-    if (!(p->tau1 >= 0.f && p->tau1 <= 1.f) || !(p->tau2 >= 0.f && p->tau2 <= 1.f))
+    if (!(p->tau1 >= 0.f && p->tau1 <= 1.f) || !(p->tau2 >= 0.f && p->tau2 <= 1.f) || p->draft_m < 0)
         return WINO_ERR_ARG;
     if (p->n_seq < 1 || p->blk_len < 1 || p->blk_len > kMaxBlkLen || p->blk_start < 0 || p->seq_len < 1 ||
         (int64_t)p->blk_start + p->blk_len > p->seq_len || p->mask_id < 0)

@@ -6,7 +6,8 @@ sequence whose block is complete is frozen (WINO_OPT_FREEZE_FINISHED): its
 own loop has ended, so it is not re-verified while the rest of the batch
 finishes the block.  The
 only device-to-host traffic per step is the [n_seq, 3] counts array, read to
-decide whether the block is finished.  The hidden states of each step come
+decide whether the block is finished (plus the token state when a trajectory
+is recorded).  The hidden states of each step come
 from a caller-supplied function (the transformer forward with the
 shadow-block attention mask is outside this library).
 """
@@ -38,7 +39,7 @@ class LoopStats:
 def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float, mask_id: int,
            hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
            on_step: Callable | None = None, last_change=None, no_shadow: bool = False,
-           compact: bool = False) -> LoopStats:
+           compact: bool = False, draft_m: int = 0, trajectory: list | None = None) -> LoopStats:
     """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
 
     ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
@@ -49,7 +50,12 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     position's WINO finalization step t_l (Sec. 5.1).  ``no_shadow``: WINO+ inference
     (Sec. 5.3): ``hidden`` returns only the n_seq*blk_len block rows, drafting uses the
     single threshold ``tau1`` and nothing is re-masked.  ``compact``: score only the row
-    each position's update reads (WINO_OPT_COMPACT), same results.
+    each position's update reads (WINO_OPT_COMPACT), same results.  ``draft_m`` > 0: draft
+    a fixed number of the most confident masked positions per step instead of Eq. 2 (naive
+    parallel sampling, Sec. 3; with ``no_shadow`` the irreversible baseline decoder, 1 =
+    greedy Eq. 1).  ``trajectory``: a list that receives the host copy of the state
+    Y^(0), Y^(1), ... (int32 [n_seq, S] arrays), one per step, for building WINO+ training
+    states (Sec. 5.1-5.2); it costs one extra device-to-host copy of ``tokens`` per step.
     """
     import torch
 
@@ -57,27 +63,40 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     d, V = int(W.shape[1]), int(W.shape[0])
     N = n_seq * (1 if (no_shadow or compact) else 2) * blk_len  # rows scored per step
     dev = tokens.device
-    p0 = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact)
+    ts = stream if stream is not None else torch.cuda.current_stream(dev)  # every copy goes on the step's stream
+    p0 = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact,
+                     draft_m=draft_m)
     ws = torch.zeros(wino_workspace_size_step(p0, d, V), dtype=torch.uint8, device=dev)
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
     counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
+    tokens_host = torch.zeros((n_seq, S), dtype=torch.int32, pin_memory=True) if trajectory is not None else None
+    if trajectory is not None:
+        with torch.cuda.stream(ts):
+            tokens_host.copy_(tokens)
+        ts.synchronize()
+        trajectory.append(tokens_host.numpy().copy())
     stats = LoopStats()
     k = 0
     for b in range(n_blocks):
         b0 = prompt_len + b * blk_len
         p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True,
-                        last_change=last_change, no_shadow=no_shadow, compact=compact)
+                        last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
         bs = BlockStats(block=b, blk_start=b0)
         while True:
             if bs.steps >= max_steps:
                 raise WinoError(WINO_ERR_MAX_STEPS, f"decode: block {b} not finished after {max_steps} steps")
             H = hidden(k, b0)
             p.step_index = k + 1
-            wino_step(H, W, tokens, p, counts, ws, flags=flags, stream=stream)
-            counts_host.copy_(counts, non_blocking=True)
-            torch.cuda.current_stream(dev).synchronize() if stream is None else stream.synchronize()
+            wino_step(H, W, tokens, p, counts, ws, flags=flags, stream=ts)
+            with torch.cuda.stream(ts):
+                counts_host.copy_(counts, non_blocking=True)
+                if tokens_host is not None:
+                    tokens_host.copy_(tokens, non_blocking=True)
+            ts.synchronize()
             c = counts_host.numpy()
+            if tokens_host is not None:
+                trajectory.append(tokens_host.numpy().copy())
             if (c < 0).any():
                 raise WinoError(int(c.min()), f"decode: device status at step {k}")
             bs.steps += 1

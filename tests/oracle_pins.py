@@ -17,7 +17,12 @@ oracle disagrees with what the paper or plain mathematics fixes:
 * an exhaustive enumeration of small states checked against the properties
   Eq. 2-4 state (drafts only on MASK, re-masks only on decoded positions,
   each draft/re-mask justified by its threshold, completeness, positions
-  outside the block untouched, counts consistent).
+  outside the block untouched, counts consistent);
+* naive parallel sampling (a fixed number M of tokens per step, Sec. 3):
+  M = 1 is Eq. 1, the drafted set is the unique size-min(M, #MASK) subset
+  that beats every left-out masked position (brute force over all subsets),
+  and a block of L_b positions takes ceil(L_b / M) steps (the 256 / 128 / 64
+  steps of Sec. 6.3.3 for 1 / 2 / 4 tokens per step).
 
 ``tests/test_oracle_pins.py`` runs them on the oracle;
 ``tests/test_oracle_mutants.py`` checks that planted mistakes fail them.
@@ -36,7 +41,7 @@ try:  # mpmath ships with sympy
 except ImportError:  # pragma: no cover
     mpmath = None
 
-MASK_FLAG = {"none": 0, "draft": 1, "fallback": 2, "remask": 3, "draft_is_mask": 4}
+MASK_FLAG = {"none": 0, "draft": 1, "fallback": 2, "remask": 3, "draft_is_mask": 4, "draft_top_m": 5}
 
 
 # ----------------------------------------------------------------------------- scoring
@@ -423,7 +428,114 @@ def pin_no_shadow_is_threshold_decoding(O):
         assert np.all(c1[:, 1] == 0)
 
 
-EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_finalization_steps, pin_no_shadow_is_threshold_decoding, pin_only_draft_never_remasks, pin_greedy_reduction,
-            pin_eq4_exhaustive_properties, pin_loop_terminates]
+def pin_fixed_m_hand_case(O):
+    """M = 2 picks the two most confident masked positions, the lower position first on ties; decoded
+    positions are verified as usual (or left alone without the shadow block)."""
+    M = 50
+    tokens = np.array([[1, M, 7, M, M, M, 8]], np.int32)  # block = positions 1..5
+    am = _rows(1, 5, [11, 12, 13, 14, 15], [0] * 5)
+    pm = _rows(1, 5, [0.25, 0.99, 0.5, 0.75, 0.5], [0.0] * 5)  # l1 is decoded: its pmax is irrelevant
+    pt = _rows(1, 5, [0.0] * 5, [0.0, 0.1, 0.0, 0.0, 0.0])
+    tok, cnt, fl = O.draft_verify(tokens, 1, 5, M, 0.0, 0.9, am, pm, pt, draft_m=2)
+    # masked l0 (0.25), l2 (0.5), l3 (0.75), l4 (0.5): l3 first, then l2 (ties with l4, lower position)
+    assert tok.tolist() == [[1, M, M, 13, 14, M, 8]], tok  # l1 re-masked: 0.1 < 0.9
+    assert cnt.tolist() == [[2, 1, 3]] and fl.tolist() == [[0, 3, 5, 5, 0]], (cnt, fl)
+    tok, cnt, fl = O.draft_verify(tokens, 1, 5, M, 0.0, 0.9, am.reshape(1, 2, 5)[:, 0].reshape(-1),
+                                  pm.reshape(1, 2, 5)[:, 0].reshape(-1), None, no_shadow=True, draft_m=2)
+    assert tok.tolist() == [[1, M, 7, 13, 14, M, 8]] and cnt.tolist() == [[2, 0, 2]], (tok, cnt)
+    # M at least the number of masks: every masked position is drafted, whatever tau1 says
+    tok, cnt, fl = O.draft_verify(tokens, 1, 5, M, 1.0, 0.0, am, pm, pt, draft_m=9)
+    assert tok.tolist() == [[1, 11, 7, 13, 14, 15, 8]] and cnt.tolist() == [[4, 0, 0]], (tok, cnt)
+
+
+def _top_m_by_sort(masked, conf, m):
+    """The drafted set of naive parallel sampling via numpy's stable sort: by confidence, then position."""
+    L = len(conf)
+    order = np.lexsort((np.arange(L), -np.where(masked, conf, -np.inf)))
+    sel = np.zeros(L, bool)
+    sel[order[:min(m, int(masked.sum()))]] = True
+    return sel & masked
+
+
+def pin_fixed_m_one_is_greedy(O):
+    """M = 1 equals the tau1 = 1 reduction (Eq. 1) step for step, and every M equals a stable sort."""
+    rng = np.random.default_rng(29)
+    n_seq, L, V, P = 24, 10, 300, 2
+    for m in (1, 2, 3, 5, 10, 12):
+        tokens = rng.integers(0, V, size=(n_seq, P + L + 2)).astype(np.int32)
+        tokens[:, P:P + L][rng.random((n_seq, L)) < 0.6] = V
+        am_b = rng.integers(0, V, size=(n_seq, L)).astype(np.int32)
+        pm_b = np.round(rng.random((n_seq, L)) * 6) / 6  # coarse grid: many exact ties
+        t1, c1, f1 = O.draft_verify(tokens, P, L, V, 0.5, 0.0, am_b.reshape(-1), pm_b.reshape(-1), None,
+                                    no_shadow=True, draft_m=m)
+        for s in range(n_seq):
+            masked = tokens[s, P:P + L] == V
+            sel = _top_m_by_sort(masked, pm_b[s], m)
+            want = np.where(sel, am_b[s], tokens[s, P:P + L])
+            assert np.array_equal(t1[s, P:P + L], want), (m, s)
+            assert np.array_equal(f1[s] == 5, sel) and c1[s, 0] == sel.sum() and c1[s, 1] == 0
+        if m == 1:
+            t2, c2, _ = O.draft_verify(tokens, P, L, V, 1.0, 0.0, am_b.reshape(-1), pm_b.reshape(-1), None,
+                                       no_shadow=True)
+            assert np.array_equal(t1, t2) and np.array_equal(c1, c2)
+
+
+def pin_fixed_m_subsets(O):
+    """Brute force over all subsets: the drafted set is the only one of size min(M, #MASK) in which every
+    member beats every masked position left out (higher confidence, or equal and a lower position)."""
+    L, V = 5, 7
+    grid = np.array([0.0, 0.5, 1.0])
+    confs = np.array(list(itertools.product(range(len(grid)), repeat=L)))  # 243 confidence patterns
+    for mask_bits in range(1 << L):
+        masked = np.array([(mask_bits >> l) & 1 for l in range(L)], bool)
+        n_seq = len(confs)
+        tokens = np.zeros((n_seq, L), np.int32)
+        tokens[:, masked] = V
+        pm_b = grid[confs]
+        am_b = np.tile(np.arange(L, dtype=np.int32), (n_seq, 1))
+        for m in (1, 2, 4):
+            tok, cnt, fl = O.draft_verify(tokens, 0, L, V, 0.5, 0.0, am_b.reshape(-1), pm_b.reshape(-1), None,
+                                          no_shadow=True, draft_m=m)
+            k = min(m, int(masked.sum()))
+            idx = np.flatnonzero(masked)
+            for s in range(0, n_seq, 7):
+                got = set(np.flatnonzero(fl[s] == 5).tolist())
+                valid = []
+                for sub in itertools.combinations(idx.tolist(), k):
+                    out = [l for l in idx if l not in sub]
+                    if all(pm_b[s, a] > pm_b[s, b] or (pm_b[s, a] == pm_b[s, b] and a < b) for a in sub for b in out):
+                        valid.append(set(sub))
+                assert len(valid) == 1 and got == valid[0], (mask_bits, m, s, got, valid)
+                assert np.array_equal(tok[s][masked & (fl[s] == 0)], np.full(int((masked & (fl[s] == 0)).sum()), V))
+
+
+def pin_fixed_m_step_count(O):
+    """A generation of 256 positions in 8 blocks of 32 takes 256 / M steps at M tokens per step
+    (256, 128 and 64 steps for 1, 2 and 4 tokens per step, Sec. 6.3.3), ceil(32 / M) per block."""
+    rng = np.random.default_rng(31)
+    n_seq, L, n_blk, V, P = 3, 32, 8, 1000, 4
+    for m, want_total in ((1, 256), (2, 128), (4, 64), (3, 8 * 11)):
+        tokens = np.full((n_seq, P + L * n_blk), V, np.int32)
+        tokens[:, :P] = 1
+        total = 0
+        for b in range(n_blk):
+            b0 = P + b * L
+            steps = 0
+            while (tokens[:, b0:b0 + L] == V).any():
+                am = rng.integers(0, V, size=n_seq * L).astype(np.int32)  # never MASK (= V)
+                pm = rng.random(n_seq * L)
+                tokens, cnt, _ = O.draft_verify(tokens, b0, L, V, 0.9, 0.9, am, pm, None, freeze_finished=True,
+                                                no_shadow=True, draft_m=m)
+                steps += 1
+                assert steps <= L
+            assert steps == -(-L // m), (m, b, steps)
+            total += steps
+        assert total == want_total, (m, total)
+        assert not (tokens == V).any()
+
+
+EQ4_PINS = [pin_eq4_hand_cases, pin_freeze_finished, pin_finalization_steps, pin_no_shadow_is_threshold_decoding,
+            pin_fixed_m_hand_case, pin_fixed_m_one_is_greedy, pin_fixed_m_subsets, pin_fixed_m_step_count,
+            pin_only_draft_never_remasks, pin_greedy_reduction, pin_eq4_exhaustive_properties, pin_loop_terminates]
 
 ALL_PINS = SCORING_PINS + EQ4_PINS

@@ -2,6 +2,8 @@
 and rejects bad arguments before touching CUDA."""
 import ctypes as C
 import re
+import shutil
+import subprocess
 from pathlib import Path
 
 import pytest
@@ -54,7 +56,7 @@ def _p(**kw):
     base = dict(tau1=0.7, tau2=0.9, mask_id=99, n_seq=2, seq_len=64, blk_start=32, blk_len=16, max_steps=10,
                 options=0)
     base.update(kw)
-    return _abi.WinoParams(*base.values())
+    return _abi.WinoParams(**base)
 
 
 def test_score_rows_argument_errors():
@@ -95,6 +97,7 @@ def test_draft_verify_argument_errors():
     assert call(_p(blk_start=50)) == wino.WINO_ERR_SHAPE  # block runs past seq_len
     assert call(_p(n_seq=0)) == wino.WINO_ERR_SHAPE
     assert call(_p(mask_id=-1)) == wino.WINO_ERR_SHAPE
+    assert call(_p(draft_m=-1)) == wino.WINO_ERR_ARG
 
 
 def test_step_argument_errors():
@@ -109,3 +112,22 @@ def test_step_argument_errors():
     assert call(_p(mask_id=100)) == wino.WINO_ERR_SHAPE  # MASK outside the vocabulary
     assert call(_p(), d=12) == wino.WINO_ERR_SHAPE
     assert call(_p(), wsb=1000) == wino.WINO_ERR_WORKSPACE
+
+
+def test_params_layout_matches_header(tmp_path):
+    """The ctypes mirror of wino_params has the C struct's size and field offsets (gcc reads the header)."""
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    fields = [f[0] for f in _abi.WinoParams._fields_]
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "wino.h"\nint main(void) {\n'
+                   '    printf("%zu\\n", sizeof(wino_params));\n' +
+                   "".join('    printf("%%zu\\n", offsetof(wino_params, %s));\n' % f for f in fields) +
+                   "    return 0;\n}\n")
+    exe = tmp_path / "layout"
+    inc = Path(__file__).resolve().parent.parent / "include"
+    subprocess.run([gcc, "-std=c11", "-I", str(inc), str(src), "-o", str(exe)], check=True)
+    got = [int(x) for x in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    assert got[0] == C.sizeof(_abi.WinoParams)
+    assert got[1:] == [getattr(_abi.WinoParams, f).offset for f in fields]

@@ -442,3 +442,96 @@ def test_decode_loop_compact_lockstep():
                         tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=500, compact=True)
     assert not np.any(host(tok_d)[:, w.prompt_len:] == w.mask_id)
     assert stats.rows_scored == stats.total_steps * w.n_seq * w.blk_len
+
+
+@pytest.mark.parametrize("n_seq,L,S,b0", CASES, ids=[f"B{c[0]}_L{c[1]}" for c in CASES])
+@pytest.mark.parametrize("m", [1, 2, 5, 2000])
+@pytest.mark.parametrize("shadow", [True, False], ids=["verify", "no_shadow"])
+def test_draft_verify_fixed_m_bit_exact(n_seq, L, S, b0, m, shadow):
+    """Fixed-M drafting (naive parallel sampling, Sec. 3) on the same fp32 statistics equals the oracle bit
+    for bit, exact ties on a coarse confidence grid included (smallest position first)."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, f32, host
+    M = 997
+    rng = np.random.default_rng(n_seq * 31 + L + m)
+    tokens, am, pm, pt = _random_case(rng, n_seq, L, S, b0, M)
+    pm = (np.round(pm * 16) / 16).astype(np.float32)
+    if not shadow:  # block rows only
+        am = am.reshape(n_seq, 2, L)[:, 0].reshape(-1).copy()
+        pm = pm.reshape(n_seq, 2, L)[:, 0].reshape(-1).copy()
+        pt = None
+    last0 = np.zeros((n_seq, S), np.int32)
+    ref_last = last0.copy()
+    ref_tok, ref_cnt, ref_fl = oracle.draft_verify(tokens, b0, L, M, f32(0.7), f32(0.9), am, pm.astype(np.float64),
+                                                   None if pt is None else pt.astype(np.float64), step_index=3,
+                                                   last_change=ref_last, no_shadow=not shadow, draft_m=m)
+    tok_d, last_d = dev(tokens), dev(last0)
+    counts = torch.full((n_seq, 3), -9, dtype=torch.int32, device="cuda")
+    flags = torch.full((n_seq, L), -9, dtype=torch.int8, device="cuda")
+    p = wino.make_params(0.7, 0.9, M, n_seq, S, b0, L, step_index=3, last_change=last_d, no_shadow=not shadow,
+                         draft_m=m)
+    wino.wino_draft_verify(tok_d, dev(am), dev(pm), None if pt is None else dev(pt), p, counts, flags)
+    torch.cuda.synchronize()
+    assert np.array_equal(host(tok_d), ref_tok)
+    assert np.array_equal(host(counts), ref_cnt) and np.array_equal(host(flags), ref_fl)
+    assert np.array_equal(host(last_d), ref_last)
+    masked = (tokens[:, b0:b0 + L] == M).sum(1)
+    assert np.array_equal(((ref_fl == 5) | (ref_fl == 4)).sum(1), np.minimum(masked, m))
+
+
+def test_decode_loop_fixed_m_lockstep():
+    """Naive parallel sampling at 2 tokens per step (no shadow block) through the loop driver with the
+    whole trajectory recorded: every step re-run by the oracle from the GPU's state, ceil(L_b / 2) steps
+    per block, and the finalization steps read off the trajectory equal the in-kernel bookkeeping."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import PROB_TOL, TIE_TOL, dev, host
+    from oracle_pins import finalization_steps_from_trajectory
+    m = 2
+    w = ws.Workload("fixed_m_loop", d=128, V=3000, n_seq=3, blk_len=32, bias=((1.0, 0.0, 8.0),), n_blocks=2,
+                    tau1=0.8, tau2=0.9, shadow=False)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    tok_d = dev(st.tokens)
+    last_d = torch.zeros_like(tok_d)
+    rec = {}
+    flagged = [0]
+    mask_drafts = [0]
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        H = ws.hidden_states(w, W, st, step=k)
+        rec["pre"], rec["H"] = host(tok_d).copy(), H
+        return dev(H)
+
+    def on_step(k, b0, counts, flags):
+        o = oracle.step(rec["H"], W, rec["pre"], b0, w.blk_len, w.mask_id, w.tau1, w.tau2, freeze_finished=True,
+                        no_shadow=True, draft_m=m)
+        got = host(tok_d)
+        L = w.blk_len
+        for s in range(w.n_seq):
+            y = rec["pre"][s, b0:b0 + L]
+            masked = y == w.mask_id
+            conf = o.pmax.reshape(w.n_seq, L)[s]
+            gap = o.gap.reshape(w.n_seq, L)[s]
+            c = np.sort(np.where(masked, conf, -np.inf))[::-1]
+            boundary_tie = masked.sum() > m and c[m - 1] - c[m] < PROB_TOL
+            diff = got[s, b0:b0 + L] != o.tokens[s, b0:b0 + L]
+            near = (masked & (gap < TIE_TOL)) | (boundary_tie & masked & (np.abs(conf - c[m - 1]) < PROB_TOL))
+            assert not (diff & ~near).any(), (k, s, np.flatnonzero(diff & ~near))
+            flagged[0] += int(near.sum())
+        mask_drafts[0] += int((host(flags) == 4).sum())
+
+    traj = []
+    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
+                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=200,
+                        last_change=last_d, no_shadow=True, draft_m=m, trajectory=traj)
+    final = host(tok_d)
+    assert not np.any(final[:, w.prompt_len:] == w.mask_id)
+    assert len(traj) == stats.total_steps + 1 and np.array_equal(traj[-1], final)
+    assert np.array_equal(traj[0], st.tokens)  # Y^(0): the state before the first step
+    assert np.array_equal(finalization_steps_from_trajectory(traj), host(last_d))
+    if mask_drafts[0] == 0:
+        assert [b.steps for b in stats.blocks] == [-(-w.blk_len // m)] * w.n_blocks
+    print("fixed-M loop steps/block", [b.steps for b in stats.blocks], "flagged", flagged[0],
+          "drafts whose argmax is MASK", mask_drafts[0])

@@ -23,7 +23,7 @@ MUTANTS = [
     ("verify_not_strict", "(ptarget[row_shd + l] < tau2)", "(ptarget[row_shd + l] <= tau2)"),
     ("draft_reads_shadow_row", "(pmax[row_blk + l] > tau1)", "(pmax[row_shd + l] > tau1)"),
     ("verify_reads_block_row", "(ptarget[row_shd + l] < tau2)", "(ptarget[row_blk + l] < tau2)"),
-    ("draft_ignores_mask_state", "inD[l] = (prev[l] == mask_id) && ", "inD[l] = "),
+    ("draft_ignores_mask_state", "(draft_m <= 0) && (prev[l] == mask_id) && ", "(draft_m <= 0) && "),
     ("verify_ignores_mask_state", "inR[l] = !no_shadow && (prev[l] != mask_id) && ", "inR[l] = !no_shadow && "),
     ("verify_runs_without_shadow", "inR[l] = !no_shadow && ", "inR[l] = "),
     ("no_fallback", "if (n_draft == 0 && n_mask > 0) {", "if (0) {"),
@@ -47,6 +47,10 @@ MUTANTS = [
     ("freeze_ignored", "if (freeze_finished && n_mask == 0) {", "if (0) {"),
     ("freeze_always", "if (freeze_finished && n_mask == 0) {", "if (n_mask == 0) {"),
     ("last_change_on_every_position", "if (last_change && y[l] != before)", "if (last_change)"),
+    ("fixed_m_last_on_ties", "pmax[row_blk + l] > pmax[row_blk + pick]", "pmax[row_blk + l] >= pmax[row_blk + pick]"),
+    ("fixed_m_one_extra", "j < draft_m && j < n_mask", "j <= draft_m && j < n_mask"),
+    ("fixed_m_keeps_threshold", "inD[l] = (draft_m <= 0) && ", "inD[l] = "),
+    ("fixed_m_ignores_mask_state", "if (prev[l] == mask_id && !inD[l] && ", "if (!inD[l] && "),
     ("last_change_off_by_one", "last_change[s * seq_len + blk_start + l] = step_index;",
      "last_change[s * seq_len + blk_start + l] = step_index - 1;"),
 ]
