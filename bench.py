@@ -243,6 +243,10 @@ def run_wino(args, rank, world, local_rank):
     import wino_synth as ws
 
     w = ws.WORKLOADS[args.workload]
+    if args.no_shadow:  # WINO+ inference: block rows only
+        import dataclasses
+        w = dataclasses.replace(w, shadow=False)
+    score_only = args.score_rows or args.entropy
     t_gen = time.time()
     W = ws.weights(w)
     st = ws.initial_state(w)
@@ -260,14 +264,21 @@ def run_wino(args, rank, world, local_rank):
     counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device=dev)
     wsp = wino.workspace(w.N, w.d, w.V, device=dev)
     p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len,
-                         compact=args.compact)
+                         compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m)
     if args.compact:  # row compaction needs room for the gathered rows
         wsp = wino.step_workspace(p, w.d, w.V, device=dev)
     stream = torch.cuda.current_stream(dev)
     sid = stream.cuda_stream
+    am = torch.empty(w.N, dtype=torch.int32, device=dev)
+    pm = torch.empty(w.N, dtype=torch.float32, device=dev)
+    pt = torch.empty(w.N, dtype=torch.float32, device=dev)
+    ent = torch.empty(w.N, dtype=torch.float32, device=dev) if args.entropy else None
 
     def step(i):
-        wino.wino_step(Hd[i % n_h], Wd, tok, p, counts, wsp, stream=sid)
+        if score_only:  # wino_score_rows alone (statistics of every row, optionally with H(p))
+            wino.wino_score_rows(Hd[i % n_h], Wd, None, am, pm, pt, wsp, stream=sid, entropy=ent)
+        else:
+            wino.wino_step(Hd[i % n_h], Wd, tok, p, counts, wsp, stream=sid)
 
     for i in range(args.warmup):
         step(i)
@@ -357,7 +368,9 @@ def run_wino(args, rank, world, local_rank):
             if pending[j]:
                 consume(j)
 
-    for i in range(max(3, args.warmup)):
+    if score_only:
+        e2e_steps = 0
+    for i in range(max(3, args.warmup) if e2e_steps else 0):
         e2e_step(i)
     e2e_drain()
     if world > 1:
@@ -369,7 +382,7 @@ def run_wino(args, rank, world, local_rank):
     e2e_drain()
     torch.cuda.synchronize(dev)
     te = time.perf_counter() - te0
-    te = job_time_max(te, world, device=dev)
+    te = job_time_max(te, world, device=dev) if e2e_steps else 0.0
     if e2e_bad[0]:
         raise RuntimeError(f"{e2e_bad[0]} end-to-end steps returned an error status")
     h2d = Hh[0].numel() * 2 + tok_h.numel() * 4
@@ -402,10 +415,19 @@ def run_wino(args, rank, world, local_rank):
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         import oracle
-        t = oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
+        if args.no_shadow or score_only:  # rows without a target
+            t = np.full(w.N, -1, np.int32)
+        else:
+            t = oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
         cpu = oracle_cpu_baseline(w, W, Hs[0], t, budget_s=args.cpu_budget_s)
 
     cfg = config_dict(w)
+    if args.no_shadow:
+        cfg["no_shadow"] = "WINO+ inference (WINO_OPT_NO_SHADOW): block rows only"
+    if args.draft_m:
+        cfg["draft_m"] = args.draft_m
+    if score_only:
+        cfg["mode"] = "wino_score_rows alone" + (" with the entropy output" if args.entropy else "")
     if args.compact:
         cfg["compact"] = "rows scored per step: %d of %d (WINO_OPT_COMPACT); value counts all %d" % (
             w.N // 2, w.N, w.N)
@@ -424,8 +446,9 @@ def run_wino(args, rank, world, local_rank):
                                                                                       peaks["bf16_tflops"])},
         "step_roofline_frac": max(t_flop, w_bytes / (peaks["hbm_gbs"] * 1e9)) / step_s,
         "tflops_per_step": flops / step_s / 1e12,
-        "e2e": {"value": job_rows_per_s(w.N, e2e_steps, world, te), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * te / e2e_steps},
+        "e2e": None if not e2e_steps else {
+            "value": job_rows_per_s(w.N, e2e_steps, world, te), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * te / e2e_steps},
         "gpu_launches": 2 * args.steps,
         "clocks": clock_info,
         "cpu_baseline": cpu,
@@ -454,6 +477,9 @@ def run_loop(args):
     import wino_synth as ws
 
     w = ws.WORKLOADS[args.workload]
+    if args.no_shadow:  # WINO+ inference: block rows only
+        import dataclasses
+        w = dataclasses.replace(w, shadow=False)
     W = ws.weights(w)
     st = ws.initial_state(w)
 
@@ -474,7 +500,7 @@ def run_loop(args):
         tok = to_dev(st.tokens)
         stats = loop.decode(Wd, tok, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks,
                             tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, max_steps=4096,
-                            compact=args.compact)
+                            compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m)
         return stats, tok
 
     t_gen = time.time()
@@ -508,6 +534,10 @@ def run_loop(args):
     if args.compact:
         line["config"]["compact"] = "rows scored per step: %d of %d (WINO_OPT_COMPACT); value counts all %d" % (
             w.N // 2, w.N, w.N)
+    if args.no_shadow:
+        line["config"]["no_shadow"] = "WINO+ inference (WINO_OPT_NO_SHADOW): block rows only"
+    if args.draft_m:
+        line["config"]["draft_m"] = args.draft_m
     print(json.dumps(line), flush=True)
 
 
@@ -522,6 +552,10 @@ def main():
     ap.add_argument("--compact", action="store_true",
                     help="row compaction: score only the row each position's update reads (not the headline: "
                          "the metric counts all 2*n_seq*blk_len rows)")
+    ap.add_argument("--no-shadow", action="store_true", help="WINO+ inference step: block rows only")
+    ap.add_argument("--draft-m", type=int, default=0, help="fixed-M drafting (naive parallel sampling)")
+    ap.add_argument("--score-rows", action="store_true", help="time wino_score_rows alone instead of the step")
+    ap.add_argument("--entropy", action="store_true", help="time wino_score_rows with the entropy output")
     ap.add_argument("--loop", action="store_true",
                     help="time the workload's whole decode loop (until no MASK is left) instead of K steps")
     ap.add_argument("--loop-repeats", type=int, default=3)
