@@ -58,7 +58,9 @@ def load_peaks():
 def config_dict(w):
     return {"workload": w.name, "N": w.N, "d": w.d, "V": w.V, "n_seq": w.n_seq, "blk_len": w.blk_len,
             "tau1": w.tau1, "tau2": w.tau2, "seed": w.seed,
-            "l2": "inputs larger than L2: W_lm is %.3f GB, read once per step" % (w.V * w.d * 2 / 1e9),
+            "l2": ("inputs larger than L2: W_lm is %.3f GB, read once per step" % (w.V * w.d * 2 / 1e9)
+                   if w.V * w.d * 2 > 129e6 else
+                   "L2-resident: W_lm is %.1f MB (a latency-bound case; L2 not flushed)" % (w.V * w.d * 2 / 1e6)),
             "parallelism": "replicas (one independent decode per GPU)"}
 
 
@@ -285,6 +287,24 @@ def run_wino(args, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     if wino.wino_read_device_status(wsp, stream=sid) != wino.WINO_OK:
         raise RuntimeError("device status not OK after warm-up")
+    run_steps = None
+    if args.graph:  # capture `graph` consecutive steps once; the timed region replays the graph
+        if args.steps % args.graph:
+            raise SystemExit("--steps must be a multiple of --graph")
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for i in range(args.graph):
+                if score_only:
+                    wino.wino_score_rows(Hd[i % n_h], Wd, None, am, pm, pt, wsp, entropy=ent)
+                else:
+                    wino.wino_step(Hd[i % n_h], Wd, tok, p, counts, wsp)
+        torch.cuda.synchronize(dev)
+
+        def run_steps(k):
+            for _ in range(k // args.graph):
+                graph.replay()
+        run_steps(args.graph)  # one untimed replay
+        torch.cuda.synchronize(dev)
 
     clocks = ClockSampler(gpu_uuid(dev)) if rank == 0 else None
     time.sleep(0.3 if clocks else 0)
@@ -296,8 +316,11 @@ def run_wino(args, rank, world, local_rank):
     # through programmatic dependent launch).
     tw0 = time.time()
     ev0.record(stream)
-    for i in range(args.steps):
-        step(i)
+    if run_steps is not None:
+        run_steps(args.steps)
+    else:
+        for i in range(args.steps):
+            step(i)
     ev1.record(stream)
     torch.cuda.synchronize(dev)
     tw1 = time.time()
@@ -428,6 +451,8 @@ def run_wino(args, rank, world, local_rank):
         cfg["draft_m"] = args.draft_m
     if score_only:
         cfg["mode"] = "wino_score_rows alone" + (" with the entropy output" if args.entropy else "")
+    if args.graph:
+        cfg["launch"] = "CUDA graph of %d consecutive steps, replayed %d times" % (args.graph, args.steps // args.graph)
     if args.compact:
         cfg["compact"] = "rows scored per step: %d of %d (WINO_OPT_COMPACT); value counts all %d" % (
             w.N // 2, w.N, w.N)
@@ -556,6 +581,8 @@ def main():
     ap.add_argument("--draft-m", type=int, default=0, help="fixed-M drafting (naive parallel sampling)")
     ap.add_argument("--score-rows", action="store_true", help="time wino_score_rows alone instead of the step")
     ap.add_argument("--entropy", action="store_true", help="time wino_score_rows with the entropy output")
+    ap.add_argument("--graph", type=int, default=0,
+                    help="capture this many consecutive steps in a CUDA graph and time its replays")
     ap.add_argument("--loop", action="store_true",
                     help="time the workload's whole decode loop (until no MASK is left) instead of K steps")
     ap.add_argument("--loop-repeats", type=int, default=3)
