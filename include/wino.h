@@ -18,6 +18,9 @@
  *     library never allocates, frees or synchronises (except
  *     wino_read_device_status, which reads back one word).
  *   - bf16 data are passed as uint16_t bit patterns (IEEE binary32 top half).
+ *   - Alignment: H and W 16 bytes, workspaces 256 bytes, int32 and float
+ *     arrays 4 bytes; a misaligned pointer is rejected with WINO_ERR_ARG
+ *     before anything is launched.
  *   - Row order of the scored rows is [s][kind][l]: sequence s, kind 0 = the
  *     current-block row of position l, kind 1 = its shadow-block row; row
  *     index n = (2*s + kind)*blk_len + l, N = 2*n_seq*blk_len.

@@ -180,6 +180,8 @@ int check_params(const wino_params *p)
         return WINO_ERR_ARG;
     if (!(p->tau1 >= 0.f && p->tau1 <= 1.f) || !(p->tau2 >= 0.f && p->tau2 <= 1.f) || p->draft_m < 0)
         return WINO_ERR_ARG;
+    if (!aligned(p->last_change, 4))
+        return WINO_ERR_ARG;
     if (p->n_seq < 1 || p->blk_len < 1 || p->blk_len > kMaxBlkLen || p->blk_start < 0 || p->seq_len < 1 ||
         (int64_t)p->blk_start + p->blk_len > p->seq_len || p->mask_id < 0)
         return WINO_ERR_SHAPE;
@@ -322,6 +324,9 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
         return WINO_ERR_ARG;
     if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign))
         return WINO_ERR_ARG;
+    if (!aligned(target, 4) || !aligned(argmax, 4) || !aligned(pmax, 4) || !aligned(ptarget, 4) ||
+        !aligned(entropy, 4))
+        return WINO_ERR_ARG;  // 32-bit elements: a misaligned pointer would fault on the device
     if (!shape_ok(N, d, V))
         return WINO_ERR_SHAPE;
     TargetSource ts{};
@@ -334,6 +339,9 @@ int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax,
                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream)
 {
     if (!tokens || !argmax || !pmax || !counts || !p || (!ptarget && !(p->options & WINO_OPT_NO_SHADOW)))
+        return WINO_ERR_ARG;
+    if (!aligned(tokens, 4) || !aligned(argmax, 4) || !aligned(pmax, 4) || !aligned(ptarget, 4) ||
+        !aligned(counts, 4))
         return WINO_ERR_ARG;
     int rc = check_params(p);
     if (rc != WINO_OK)
@@ -352,7 +360,7 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
 {
     if (!H || !W || !tokens || !counts || !ws)
         return WINO_ERR_ARG;
-    if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign))
+    if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign) || !aligned(tokens, 4) || !aligned(counts, 4))
         return WINO_ERR_ARG;
     int rc = check_params(p);
     if (rc != WINO_OK)

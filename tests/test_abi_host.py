@@ -71,6 +71,10 @@ def test_score_rows_argument_errors():
     for k in ("H", "W", "a", "pm", "pt", "ws"):
         assert call(**{k: None}) == wino.WINO_ERR_ARG, k
     assert call(H=FAKE + 2) == wino.WINO_ERR_ARG
+    for k in ("a", "pm", "pt"):
+        assert call(**{k: FAKE + 2}) == wino.WINO_ERR_ARG, k
+    assert call(t=FAKE + 1) == wino.WINO_ERR_ARG
+    assert call(ent=FAKE + 6) == wino.WINO_ERR_ARG
     assert call(W=FAKE + 8) == wino.WINO_ERR_ARG
     assert call(ws=FAKE + 16) == wino.WINO_ERR_ARG
     assert call(d=60) == wino.WINO_ERR_SHAPE
@@ -98,6 +102,9 @@ def test_draft_verify_argument_errors():
     assert call(_p(n_seq=0)) == wino.WINO_ERR_SHAPE
     assert call(_p(mask_id=-1)) == wino.WINO_ERR_SHAPE
     assert call(_p(draft_m=-1)) == wino.WINO_ERR_ARG
+    for k in ("tok", "am", "pm", "pt", "cnt"):
+        assert call(_p(), **{k: FAKE + 2}) == wino.WINO_ERR_ARG, k
+    assert call(_p(last_change=FAKE + 3)) == wino.WINO_ERR_ARG
 
 
 def test_step_argument_errors():
@@ -112,6 +119,9 @@ def test_step_argument_errors():
     assert call(_p(mask_id=100)) == wino.WINO_ERR_SHAPE  # MASK outside the vocabulary
     assert call(_p(), d=12) == wino.WINO_ERR_SHAPE
     assert call(_p(), wsb=1000) == wino.WINO_ERR_WORKSPACE
+    assert call(_p(), tok=FAKE + 2) == wino.WINO_ERR_ARG
+    assert call(_p(), cnt=FAKE + 1) == wino.WINO_ERR_ARG
+    assert call(_p(last_change=FAKE + 2)) == wino.WINO_ERR_ARG
 
 
 def test_params_layout_matches_header(tmp_path):
