@@ -64,7 +64,7 @@ def build(force: bool = False, verbose: bool = False, extra: list[str] | None = 
     with ThreadPoolExecutor(max(1, min(8, os.cpu_count() or 1))) as ex:
         objs = list(ex.map(compile_one, sources()))
     tmp = LIB.with_suffix(f".so.tmp{os.getpid()}")
-    cmd = [cc, *ARCH, "-shared", "-o", str(tmp), *map(str, objs)]
+    cmd = [cc, *ARCH, "-shared", "-o", str(tmp), *map(str, objs), "-ldl"]  # -ldl: NVTX loads its tool
     r = subprocess.run(cmd, capture_output=True, text=True)
     if verbose or r.returncode != 0:
         print(" ".join(cmd), r.stdout, r.stderr, sep="\n", file=sys.stderr)

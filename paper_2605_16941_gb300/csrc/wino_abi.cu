@@ -10,6 +10,7 @@
 #include <mutex>
 
 #include <cudaTypedefs.h>  // PFN_cuTensorMapEncodeTiled
+#include <nvtx3/nvToolsExt.h>
 
 #include "internal.h"
 
@@ -148,6 +149,17 @@ int tensor_map(const void *ptr, int64_t rows, int64_t cols, int box_rows, CUtens
     *out = m;
     return WINO_OK;
 }
+
+// ---------------------------------------------------------------- tracing
+
+// A named range around each entry point for timeline tools (Nsight Systems, ncu --nvtx); NVTX v3 is
+// header-only and a range costs a few nanoseconds when no tool is attached.
+struct Range {
+    explicit Range(const char *name) { nvtxRangePushA(name); }
+    ~Range() { nvtxRangePop(); }
+    Range(const Range &) = delete;
+    Range &operator=(const Range &) = delete;
+};
 
 // ---------------------------------------------------------------- launch timing
 
@@ -320,6 +332,7 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
                     int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws, size_t ws_bytes,
                     void *stream)
 {
+    const Range range("wino_score_rows");
     if (!H || !W || !argmax || !pmax || !ptarget || !ws)
         return WINO_ERR_ARG;
     if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign))
@@ -338,6 +351,7 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
 int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream)
 {
+    const Range range("wino_draft_verify");
     if (!tokens || !argmax || !pmax || !counts || !p || (!ptarget && !(p->options & WINO_OPT_NO_SHADOW)))
         return WINO_ERR_ARG;
     if (!aligned(tokens, 4) || !aligned(argmax, 4) || !aligned(pmax, 4) || !aligned(ptarget, 4) ||
@@ -358,6 +372,7 @@ int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax,
 int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
               int32_t *counts, int8_t *flags, void *ws, size_t ws_bytes, void *stream)
 {
+    const Range range("wino_step");
     if (!H || !W || !tokens || !counts || !ws)
         return WINO_ERR_ARG;
     if (!aligned(H, 16) || !aligned(W, 16) || !aligned(ws, kAlign) || !aligned(tokens, 4) || !aligned(counts, 4))

@@ -32,14 +32,27 @@ class BlockStats:
 @dataclass
 class LoopStats:
     blocks: list = field(default_factory=list)
-    total_steps: int = 0
+    total_steps: int = 0  # steps this call ran
     rows_scored: int = 0
+    next_step: int = 0  # global index of the step after the last one run
+
+
+def resume_point(k: int, blk_start: int, counts, *, prompt_len: int, blk_len: int) -> tuple[int, int]:
+    """(start_block, start_step) that continue a decode after its global step ``k``, from the arguments
+    ``on_step`` receives.  A checkpoint of a decode is the token state (and ``last_change``) after step
+    ``k`` together with this pair: the hidden states of later steps depend only on the step index and
+    the block, so a decode resumed from it replays the uninterrupted one exactly."""
+    import numpy as np
+    b = (blk_start - prompt_len) // blk_len
+    done = bool((np.asarray(counts)[:, 2] == 0).all())
+    return (b + 1 if done else b), k + 1
 
 
 def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float, mask_id: int,
            hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
            on_step: Callable | None = None, last_change=None, no_shadow: bool = False,
-           compact: bool = False, draft_m: int = 0, trajectory: list | None = None) -> LoopStats:
+           compact: bool = False, draft_m: int = 0, trajectory: list | None = None, start_block: int = 0,
+           start_step: int = 0) -> LoopStats:
     """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
 
     ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
@@ -56,6 +69,8 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     greedy Eq. 1).  ``trajectory``: a list that receives the host copy of the state
     Y^(0), Y^(1), ... (int32 [n_seq, S] arrays), one per step, for building WINO+ training
     states (Sec. 5.1-5.2); it costs one extra device-to-host copy of ``tokens`` per step.
+    ``start_block``, ``start_step``: resume a checkpointed decode (see ``resume_point``): blocks
+    before ``start_block`` are taken as done and the global step count starts at ``start_step``.
     """
     import torch
 
@@ -77,8 +92,8 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
         ts.synchronize()
         trajectory.append(tokens_host.numpy().copy())
     stats = LoopStats()
-    k = 0
-    for b in range(n_blocks):
+    k = start_step
+    for b in range(start_block, n_blocks):
         b0 = prompt_len + b * blk_len
         p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True,
                         last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
@@ -109,5 +124,6 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
             if (c[:, 2] == 0).all():
                 break
         stats.blocks.append(bs)
-    stats.total_steps = k
+    stats.total_steps = k - start_step
+    stats.next_step = k
     return stats

@@ -535,3 +535,50 @@ def test_decode_loop_fixed_m_lockstep():
         assert [b.steps for b in stats.blocks] == [-(-w.blk_len // m)] * w.n_blocks
     print("fixed-M loop steps/block", [b.steps for b in stats.blocks], "flagged", flagged[0],
           "drafts whose argmax is MASK", mask_drafts[0])
+
+
+def test_decode_loop_checkpoint_resume():
+    """A decode interrupted after a step and resumed from its checkpoint (token state, finalization
+    bookkeeping, resume point) ends in the same state as the uninterrupted decode, with the same steps,
+    whether the interruption falls inside a block or at a block's last step."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import dev, host
+    w = ws.Workload("resume", d=64, V=1000, n_seq=3, blk_len=8, bias=((1.0, 2.0, 6.0),), n_blocks=3,
+                    bias_step=0.5, tau1=0.7, tau2=0.9)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+
+    def hidden(k, b0):
+        st.blk_start = b0
+        return dev(ws.hidden_states(w, W, st, step=k))
+
+    kw = dict(prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1, tau2=w.tau2,
+              mask_id=w.mask_id, hidden=hidden, max_steps=400)
+    tok_a, last_a = dev(st.tokens), torch.zeros_like(dev(st.tokens))
+    ends = []  # per step: did it finish its block?
+    full = loop.decode(Wd, tok_a, last_change=last_a,
+                       on_step=lambda k, b0, c, f: ends.append(bool((c[:, 2] == 0).all())), **kw)
+    block_ends = [k for k, e in enumerate(ends) if e]
+    assert len(block_ends) == w.n_blocks and full.next_step == full.total_steps
+    for stop_at in sorted({3, block_ends[0], block_ends[1] - 1}):
+
+        class Stop(Exception):
+            pass
+
+        saved = {}
+
+        def on_step(k, b0, counts, flags):
+            if k == stop_at:
+                saved["tok"], saved["last"] = host(tok_b).copy(), host(last_b).copy()
+                saved["at"] = loop.resume_point(k, b0, counts, prompt_len=w.prompt_len, blk_len=w.blk_len)
+                raise Stop
+
+        tok_b, last_b = dev(st.tokens), torch.zeros_like(dev(st.tokens))
+        with pytest.raises(Stop):
+            loop.decode(Wd, tok_b, last_change=last_b, on_step=on_step, **kw)
+        start_block, start_step = saved["at"]
+        tok_c, last_c = dev(saved["tok"]), dev(saved["last"])
+        rest = loop.decode(Wd, tok_c, last_change=last_c, start_block=start_block, start_step=start_step, **kw)
+        assert np.array_equal(host(tok_c), host(tok_a)) and np.array_equal(host(last_c), host(last_a)), stop_at
+        assert start_step + rest.total_steps == full.total_steps and rest.next_step == full.next_step
