@@ -31,6 +31,7 @@ from __future__ import annotations
 
 import itertools
 from fractions import Fraction
+from pathlib import Path
 
 import numpy as np
 
@@ -509,12 +510,28 @@ def pin_fixed_m_subsets(O):
                 assert np.array_equal(tok[s][masked & (fl[s] == 0)], np.full(int((masked & (fl[s] == 0)).sum()), V))
 
 
+GOLDEN = Path(__file__).resolve().parent / "golden"
+
+
+def naive_parallel_steps():
+    """(gen_len, blk_len, tokens_per_step, steps) rows printed in Sec. 6.3.3 (tests/golden)."""
+    rows = []
+    for line in (GOLDEN / "naive_parallel_steps.txt").read_text().splitlines():
+        if line.strip() and not line.startswith("#"):
+            rows.append(tuple(int(x) for x in line.split()))
+    return rows
+
+
 def pin_fixed_m_step_count(O):
-    """A generation of 256 positions in 8 blocks of 32 takes 256 / M steps at M tokens per step
-    (256, 128 and 64 steps for 1, 2 and 4 tokens per step, Sec. 6.3.3), ceil(32 / M) per block."""
+    """The paper's step counts for a fixed number of tokens per step (Sec. 6.3.3: a generation of 256 in
+    blocks of 128 takes 256, 128 and 64 steps at 1, 2 and 4 tokens per step), and ceil(L_b / M) per block
+    for other splits (8 blocks of 32, M = 3: 8 x 11 steps)."""
     rng = np.random.default_rng(31)
-    n_seq, L, n_blk, V, P = 3, 32, 8, 1000, 4
-    for m, want_total in ((1, 256), (2, 128), (4, 64), (3, 8 * 11)):
+    cases = [(gen // blk, blk, m, steps) for gen, blk, m, steps in naive_parallel_steps()]
+    assert len(cases) == 3
+    cases.append((8, 32, 3, 8 * 11))
+    for n_blk, L, m, want_total in cases:
+        n_seq, V, P = 3, 1000, 4
         tokens = np.full((n_seq, P + L * n_blk), V, np.int32)
         tokens[:, :P] = 1
         total = 0
