@@ -474,7 +474,7 @@ def run_wino(args, rank, world, local_rank):
         "e2e": None if not e2e_steps else {
             "value": job_rows_per_s(w.N, e2e_steps, world, te), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * te / e2e_steps},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": (3 if args.compact and not score_only else 2) * args.steps,  # (gather +) score + finish
         "clocks": clock_info,
         "cpu_baseline": cpu,
     }
