@@ -122,16 +122,18 @@ class ClockSampler:
 
 def ncu_traffic(workload_name: str):
     """DRAM bytes per score launch from the committed ncu capture, if it was taken on this workload and
-    the score kernel's source has not changed since (else None)."""
+    none of the score kernel's source files has changed since (else None)."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "score_kernel_traffic.txt")) as f:
             rec = json.load(f)
-        with open(os.path.join(ROOT, "paper_2605_16941_gb300", "csrc", "score.cu"), "rb") as f:
-            h = hashlib.sha256(f.read()).hexdigest()[:16]
-    except (OSError, ValueError):
+        h = hashlib.sha256()
+        for name in rec["score_kernel_sources"]:
+            with open(os.path.join(ROOT, "paper_2605_16941_gb300", "csrc", name), "rb") as f:
+                h.update(f.read())
+    except (OSError, ValueError, KeyError, TypeError):
         return None
-    if rec.get("workload") != workload_name or rec.get("score_cu_sha256_prefix") != h:
+    if rec.get("workload") != workload_name or rec.get("sources_sha256_prefix") != h.hexdigest()[:16]:
         return None
     return float(rec["dram_bytes_read"]) + float(rec["dram_bytes_write"])
 
