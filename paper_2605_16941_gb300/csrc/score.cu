@@ -29,6 +29,8 @@
 // abort flag, records WINO_ERR_DEVICE_TIMEOUT in the status word, drains its
 // in-flight copies and MMAs (again bounded); both CTAs then meet at the
 // closing cluster barrier before TMEM is released.
+#include <mutex>
+
 #include "internal.h"
 #include "ptx.cuh"
 #include "wait.cuh"
@@ -408,11 +410,13 @@ cudaLaunchConfig_t score_config(unsigned grid, cudaStream_t stream, cudaLaunchAt
 // Per-device one-time set-up: shared-memory opt-in and the number of co-resident pairs.
 int configure_device()
 {
+    static std::mutex mu;
     static int pairs[64];
     static bool done[64];
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
         return -1;
+    std::lock_guard<std::mutex> g(mu);
     if (!done[dev]) {
         if (cudaFuncSetAttribute(score_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kScoreSmemBytes) != cudaSuccess ||
