@@ -57,7 +57,8 @@ typedef enum {
     WINO_OK = 0,
     WINO_ERR_ARG = -1,            /* null pointer, misaligned pointer, threshold out of range  */
     WINO_ERR_SHAPE = -2,          /* sizes outside the supported range (see each call)         */
-    WINO_ERR_WORKSPACE = -3,      /* ws_bytes below wino_workspace_size()                      */
+    WINO_ERR_WORKSPACE = -3,      /* ws_bytes below wino_workspace_size(), or a problem larger
+                                     than the fixed array of wino_step_static_scratch          */
     WINO_ERR_CUDA = -4,           /* a CUDA runtime/driver call or kernel launch failed        */
     WINO_ERR_MAX_STEPS = -5,      /* a decode loop exceeded its step budget (loop drivers)     */
     WINO_ERR_DEVICE_TIMEOUT = -6, /* a bounded device-side wait expired; outputs are invalid   */
