@@ -523,11 +523,13 @@ def run_loop(args):
             cache[k] = to_dev(ws.hidden_states(w, W, st, step=k))
         return cache[k]
 
+    driver = loop.decode if args.python_loop else loop.decode_native
+
     def run():
         tok = to_dev(st.tokens)
-        stats = loop.decode(Wd, tok, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks,
-                            tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, max_steps=4096,
-                            compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m)
+        stats = driver(Wd, tok, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks,
+                       tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, max_steps=4096,
+                       compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m)
         return stats, tok
 
     t_gen = time.time()
@@ -556,7 +558,8 @@ def run_loop(args):
                  "remasked_per_block": [b.remasked for b in stats.blocks],
                  "total_steps": stats.total_steps, "repeats": len(runs),
                  "timing": "wall clock around the whole decode (median of the repeats); hidden states resident "
-                           "in device memory; includes the per-step counts read-back the loop needs"},
+                           "in device memory; includes the per-step counts read-back the loop needs",
+                 "driver": "Python loop (loop.decode)" if args.python_loop else "library loop (wino_decode)"},
     }
     if args.compact:
         line["config"]["compact"] = "rows scored per step: %d of %d (WINO_OPT_COMPACT); value counts all %d" % (
@@ -588,6 +591,8 @@ def main():
     ap.add_argument("--loop", action="store_true",
                     help="time the workload's whole decode loop (until no MASK is left) instead of K steps")
     ap.add_argument("--loop-repeats", type=int, default=3)
+    ap.add_argument("--python-loop", action="store_true",
+                    help="with --loop: step from the Python driver (loop.decode) instead of the library's loop")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     ap.add_argument("--ref-budget-s", type=float, default=90.0)
     args = ap.parse_args()

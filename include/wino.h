@@ -14,9 +14,10 @@
  *   - everything else, and every position outside the block, is unchanged.
  *
  * Conventions shared by every entry point
- *   - Every array argument is a DEVICE pointer owned by the caller; the
- *     library never allocates, frees or synchronises (except
- *     wino_read_device_status, which reads back one word).
+ *   - Every array argument is a DEVICE pointer owned by the caller unless
+ *     marked host; the library never allocates, frees or synchronises
+ *     (except wino_read_device_status, which reads back one word, and
+ *     wino_decode, whose loop reads each step's counts back).
  *   - bf16 data are passed as uint16_t bit patterns (IEEE binary32 top half).
  *   - Alignment: H and W 16 bytes, workspaces 256 bytes, int32 and float
  *     arrays 4 bytes; a misaligned pointer is rejected with WINO_ERR_ARG
@@ -74,7 +75,7 @@ typedef struct {
     int32_t seq_len;   /* S: length of each row of `tokens`                                      */
     int32_t blk_start; /* first position of the current block Y_cur                             */
     int32_t blk_len;   /* L_b, 1..1024; blk_start + blk_len <= seq_len                           */
-    int32_t max_steps; /* step budget for loop drivers; unused by the calls below               */
+    int32_t max_steps; /* step budget per block for loop drivers (wino_decode); unused elsewhere */
     int32_t options;   /* bit set of WINO_OPT_* below; 0 = plain Eq. 4 on every sequence        */
     int32_t step_index;   /* k, the index of the state this step produces (Y^(k)); see last_change */
     int32_t *last_change; /* optional device int32 [n_seq, seq_len]: every position whose token the
@@ -217,6 +218,40 @@ WINO_API int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t 
 #define WINO_STATIC_SCRATCH_BYTES (16u << 20)
 WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens,
                                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream);
+
+/*
+ * Semi-autoregressive WINO decode (Sec. 3 and Sec. 4.2.3) run by the library:
+ * blocks first_block .. n_blocks-1 are decoded left to right, block b starting
+ * at position p->blk_start + b * p->blk_len; each block is stepped with
+ * wino_step until none of its positions is MASK in any sequence.  The
+ * hidden states of every step come from the caller (the transformer forward
+ * with the shadow-block attention mask is outside this library):
+ *   hidden(user, k, blk_start) returns the device bf16 rows of global step k
+ *   for the block at blk_start, laid out as wino_step's H, and must stay
+ *   valid until the next call of `hidden` or the return of wino_decode;
+ *   NULL stops the decode with WINO_ERR_ARG.
+ * Step k (counted from first_step) produces state Y^(k+1): it runs with
+ * p->step_index = k + 1 (see last_change).  After every step the [n_seq, 3]
+ * counts are copied to counts_host (host memory, pinned for speed) and the
+ * stream is synchronised to decide whether the block is done: this call
+ * blocks the calling thread.  p->options apply to every step; batched
+ * decodes want WINO_OPT_FREEZE_FINISHED.  A block that is still not done
+ * after p->max_steps (>= 1) steps returns WINO_ERR_MAX_STEPS; a device
+ * failure returns its status (tokens then hold the last good state).
+ *   block_stats  host [n_blocks] or NULL: per block {steps, drafted, re-masked}
+ *                (entries before first_block untouched)
+ *   next_step    host or NULL: the global index after the last step run;
+ *                with the block that follows, the point to resume from
+ * counts, flags (optional), ws and ws_bytes are as for wino_step.
+ */
+typedef const uint16_t *(*wino_hidden_fn)(void *user, int32_t step, int32_t blk_start);
+typedef struct {
+    int32_t steps, drafted, remasked;
+} wino_block_stats;
+WINO_API int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
+                         int32_t n_blocks, int32_t first_block, int32_t first_step, wino_hidden_fn hidden,
+                         void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, void *ws,
+                         size_t ws_bytes, void *stream, wino_block_stats *block_stats, int32_t *next_step);
 
 /*
  * Waits for `stream`, then reads the workspace status word written by the

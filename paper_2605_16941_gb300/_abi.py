@@ -33,7 +33,7 @@ WINO_OPT_COMPACT = 4
 
 EXPORTS = ("wino_workspace_size", "wino_workspace_size_step", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
-           "wino_selftest_wait_timeout", "wino_status_string", "wino_version")
+           "wino_selftest_wait_timeout", "wino_status_string", "wino_version", "wino_decode")
 
 # size of the fixed device array behind wino_step_static_scratch
 WINO_STATIC_SCRATCH_BYTES = 16 << 20
@@ -50,6 +50,14 @@ class WinoParams(C.Structure):
                 ("seq_len", C.c_int32), ("blk_start", C.c_int32), ("blk_len", C.c_int32),
                 ("max_steps", C.c_int32), ("options", C.c_int32), ("step_index", C.c_int32),
                 ("last_change", C.c_void_p), ("draft_m", C.c_int32)]
+
+
+class WinoBlockStats(C.Structure):
+    _fields_ = [("steps", C.c_int32), ("drafted", C.c_int32), ("remasked", C.c_int32)]
+
+
+# const uint16_t *(*)(void *user, int32_t step, int32_t blk_start)
+HIDDEN_FN = C.CFUNCTYPE(C.c_void_p, C.c_void_p, C.c_int32, C.c_int32)
 
 
 def library_path() -> Path:
@@ -88,6 +96,10 @@ def lib() -> C.CDLL:
         L.wino_status_string.argtypes = [C.c_int]
         L.wino_version.restype = C.c_int
         L.wino_version.argtypes = []
+        L.wino_decode.restype = C.c_int
+        L.wino_decode.argtypes = [vp, i64, i64, vp, C.POINTER(WinoParams), C.c_int32, C.c_int32, C.c_int32,
+                                  HIDDEN_FN, vp, vp, vp, vp, vp, sz, vp, C.POINTER(WinoBlockStats),
+                                  C.POINTER(C.c_int32)]
         _lib = L
     return _lib
 
@@ -191,6 +203,38 @@ def wino_step_static_scratch(H, W, tokens, params: WinoParams, counts, flags=Non
     V = int(W.shape[0]) if V is None else V
     _check(lib().wino_step_static_scratch(_ptr(H), _ptr(W), d, V, _ptr(tokens), C.byref(params), _ptr(counts),
                                           _ptr(flags), _stream(stream)), "wino_step_static_scratch")
+
+
+def wino_decode(W, tokens, params: WinoParams, n_blocks: int, hidden, counts, counts_host, ws, flags=None,
+                stream=None, *, first_block: int = 0, first_step: int = 0, d: int | None = None,
+                V: int | None = None):
+    """The library's decode loop (wino_decode).  ``hidden(k, blk_start)`` returns step k's device bf16
+    hidden states (a tensor, kept alive until the next call); ``counts_host`` is a host int32 [n_seq, 3]
+    tensor (pinned for speed).  Returns (status, per-block stats list, next step index); the status is
+    WINO_OK or the error that stopped the loop (an exception raised by ``hidden`` is re-raised)."""
+    d = int(W.shape[1]) if d is None else d
+    V = int(W.shape[0]) if V is None else V
+    held, failure = [None], []
+
+    def cb(user, k, blk_start):
+        try:
+            H = hidden(int(k), int(blk_start))
+            held[0] = H
+            return _ptr(H)
+        except BaseException as e:  # reported after the call: an exception cannot cross the C frame
+            failure.append(e)
+            return None
+
+    fn = HIDDEN_FN(cb)
+    stats = (WinoBlockStats * n_blocks)()
+    nxt = C.c_int32(0)
+    ws_bytes = ws.numel() * ws.element_size()
+    rc = lib().wino_decode(_ptr(W), d, V, _ptr(tokens), C.byref(params), n_blocks, first_block, first_step, fn,
+                           None, _ptr(counts), _ptr(counts_host), _ptr(flags), _ptr(ws), ws_bytes, _stream(stream),
+                           stats, C.byref(nxt))
+    if failure:
+        raise failure[0]
+    return rc, [(b.steps, b.drafted, b.remasked) for b in stats], nxt.value
 
 
 def wino_read_device_status(ws, stream=None) -> int:

@@ -1,0 +1,79 @@
+// decode.cu -- the semi-autoregressive decode loop (Sec. 3 and Sec. 4.2.3) run by the library.
+//
+// Blocks are decoded left to right; inside a block wino_step is repeated until
+// no position of the block is MASK in any sequence.  The hidden states of each
+// step come from a caller callback (the transformer forward is outside this
+// library); after each step the [n_seq, 3] counts are copied to the caller's
+// host buffer and the stream is synchronised, because whether the block is done
+// is only known once the step has run.  The loop is host code only: every
+// launch goes through wino_step.
+#include <cuda_runtime.h>
+
+#include "trace.h"
+#include "wino.h"
+
+extern "C" int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
+                           int32_t n_blocks, int32_t first_block, int32_t first_step, wino_hidden_fn hidden,
+                           void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, void *ws,
+                           size_t ws_bytes, void *stream, wino_block_stats *block_stats, int32_t *next_step)
+{
+    const wino::Range range("wino_decode");
+    if (!W || !tokens || !p || !hidden || !counts || !counts_host || !ws)
+        return WINO_ERR_ARG;
+    if (n_blocks < 1 || first_block < 0 || first_block > n_blocks || first_step < 0 || p->max_steps < 1)
+        return WINO_ERR_ARG;
+    if (p->n_seq < 1 || p->blk_len < 1 || p->blk_start < 0 ||
+        (int64_t)p->blk_start + (int64_t)n_blocks * p->blk_len > (int64_t)p->seq_len)
+        return WINO_ERR_SHAPE;  // every block must lie inside the sequence
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t count_bytes = (size_t)p->n_seq * 3 * sizeof(int32_t);
+    wino_params q = *p;
+    int32_t k = first_step;
+    int rc = WINO_OK;
+    for (int32_t b = first_block; b < n_blocks && rc == WINO_OK; ++b) {
+        q.blk_start = p->blk_start + b * p->blk_len;
+        wino_block_stats bs{0, 0, 0};
+        for (;;) {
+            if (bs.steps >= p->max_steps) {
+                rc = WINO_ERR_MAX_STEPS;
+                break;
+            }
+            const uint16_t *H = hidden(user, k, q.blk_start);
+            if (!H) {
+                rc = WINO_ERR_ARG;
+                break;
+            }
+            q.step_index = k + 1;  // this step produces state Y^(k+1)
+            rc = wino_step(H, W, d, V, tokens, &q, counts, flags, ws, ws_bytes, stream);
+            if (rc != WINO_OK)
+                break;
+            if (cudaMemcpyAsync(counts_host, counts, count_bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+                cudaStreamSynchronize(s) != cudaSuccess) {
+                rc = WINO_ERR_CUDA;
+                break;
+            }
+            bool done = true;
+            for (int32_t i = 0; i < p->n_seq; ++i) {
+                const int32_t *c = counts_host + 3 * i;
+                if (c[0] < 0 || c[1] < 0 || c[2] < 0) {  // a device failure: the state was left alone
+                    rc = c[0] < 0 ? c[0] : (c[1] < 0 ? c[1] : c[2]);
+                    break;
+                }
+                bs.drafted += c[0];
+                bs.remasked += c[1];
+                done = done && c[2] == 0;
+            }
+            if (rc != WINO_OK)
+                break;
+            ++k;
+            ++bs.steps;
+            if (done)
+                break;
+        }
+        if (block_stats)
+            block_stats[b] = bs;
+    }
+    if (next_step)
+        *next_step = k;
+    return rc;
+}

@@ -10,9 +10,9 @@
 #include <mutex>
 
 #include <cudaTypedefs.h>  // PFN_cuTensorMapEncodeTiled
-#include <nvtx3/nvToolsExt.h>
 
 #include "internal.h"
+#include "trace.h"
 
 namespace wino {
 namespace {
@@ -149,17 +149,6 @@ int tensor_map(const void *ptr, int64_t rows, int64_t cols, int box_rows, CUtens
     *out = m;
     return WINO_OK;
 }
-
-// ---------------------------------------------------------------- tracing
-
-// A named range around each entry point for timeline tools (Nsight Systems, ncu --nvtx); NVTX v3 is
-// header-only and a range costs a few nanoseconds when no tool is attached.
-struct Range {
-    explicit Range(const char *name) { nvtxRangePushA(name); }
-    ~Range() { nvtxRangePop(); }
-    Range(const Range &) = delete;
-    Range &operator=(const Range &) = delete;
-};
 
 // ---------------------------------------------------------------- launch timing
 

@@ -16,7 +16,8 @@ from __future__ import annotations
 from dataclasses import dataclass, field
 from typing import Callable
 
-from ._abi import WINO_ERR_MAX_STEPS, WinoError, make_params, wino_step, wino_workspace_size_step
+from ._abi import (WINO_ERR_MAX_STEPS, WINO_OK, WinoError, make_params, wino_decode, wino_step,
+                   wino_workspace_size_step)
 
 
 @dataclass
@@ -126,4 +127,39 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
         stats.blocks.append(bs)
     stats.total_steps = k - start_step
     stats.next_step = k
+    return stats
+
+
+def decode_native(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float,
+                  mask_id: int, hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
+                  last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0,
+                  start_block: int = 0, start_step: int = 0) -> LoopStats:
+    """``decode`` with the step loop run by the library (``wino_decode``): the same steps, states and
+    statistics, with one callback into Python per step (for the hidden states) instead of the whole
+    per-step bookkeeping.  No ``on_step`` or ``trajectory``; errors raise ``WinoError``."""
+    import torch
+
+    n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
+    d, V = int(W.shape[1]), int(W.shape[0])
+    N = n_seq * (1 if (no_shadow or compact) else 2) * blk_len
+    dev = tokens.device
+    ts = stream if stream is not None else torch.cuda.current_stream(dev)
+    p = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, max_steps, freeze_finished=True,
+                    last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
+    ws = torch.zeros(wino_workspace_size_step(p, d, V), dtype=torch.uint8, device=dev)
+    counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
+    counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
+    torch.cuda.current_stream(dev).synchronize()  # the buffers above are ready before the library's stream runs
+    rc, blocks, nxt = wino_decode(W, tokens, p, n_blocks, hidden, counts, counts_host, ws, stream=ts,
+                                  first_block=start_block, first_step=start_step)
+    if rc != WINO_OK:
+        raise WinoError(rc, f"wino_decode (stopped at step {nxt})")
+    stats = LoopStats()
+    for b in range(start_block, n_blocks):
+        steps, drafted, remasked = blocks[b]
+        stats.blocks.append(BlockStats(block=b, blk_start=prompt_len + b * blk_len, steps=steps, drafted=drafted,
+                                       remasked=remasked))
+    stats.total_steps = nxt - start_step
+    stats.rows_scored = N * stats.total_steps
+    stats.next_step = nxt
     return stats

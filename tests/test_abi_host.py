@@ -141,3 +141,28 @@ def test_params_layout_matches_header(tmp_path):
     got = [int(x) for x in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
     assert got[0] == C.sizeof(_abi.WinoParams)
     assert got[1:] == [getattr(_abi.WinoParams, f).offset for f in fields]
+
+
+def test_decode_argument_errors():
+    """wino_decode refuses bad arguments before calling the hidden-state callback or launching anything."""
+    L = wino.lib()
+    called = []
+    fn = _abi.HIDDEN_FN(lambda user, k, b0: called.append(k) or FAKE)
+    host = (C.c_int32 * 6)()
+
+    def call(p, n_blocks=2, first_block=0, first_step=0, hidden=fn, **kw):
+        a = dict(W=FAKE, tok=FAKE, cnt=FAKE, cnth=C.addressof(host), ws=FAKE)
+        a.update(kw)
+        return L.wino_decode(a["W"], 64, 100, a["tok"], C.byref(p) if p is not None else None, n_blocks,
+                             first_block, first_step, hidden, None, a["cnt"], a["cnth"], None, a["ws"], 1 << 30,
+                             None, None, None)
+    for k in ("W", "tok", "cnt", "cnth", "ws"):
+        assert call(_p(), **{k: None}) == wino.WINO_ERR_ARG, k
+    assert call(None) == wino.WINO_ERR_ARG
+    assert call(_p(), hidden=_abi.HIDDEN_FN()) == wino.WINO_ERR_ARG  # null callback
+    assert call(_p(), n_blocks=0) == wino.WINO_ERR_ARG
+    assert call(_p(), first_block=3) == wino.WINO_ERR_ARG
+    assert call(_p(), first_step=-1) == wino.WINO_ERR_ARG
+    assert call(_p(max_steps=0)) == wino.WINO_ERR_ARG
+    assert call(_p(), n_blocks=3) == wino.WINO_ERR_SHAPE  # blocks 32..80 run past seq_len 64
+    assert called == []
