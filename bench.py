@@ -556,6 +556,7 @@ def run_loop(args):
                  "steps_per_block": [b.steps for b in stats.blocks],
                  "drafted_per_block": [b.drafted for b in stats.blocks],
                  "remasked_per_block": [b.remasked for b in stats.blocks],
+                 "fallback_drafts_per_block": [b.fallback for b in stats.blocks],
                  "total_steps": stats.total_steps, "repeats": len(runs),
                  "timing": "wall clock around the whole decode (median of the repeats); hidden states resident "
                            "in device memory; includes the per-step counts read-back the loop needs",

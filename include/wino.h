@@ -238,20 +238,24 @@ WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int6
  * decodes want WINO_OPT_FREEZE_FINISHED.  A block that is still not done
  * after p->max_steps (>= 1) steps returns WINO_ERR_MAX_STEPS; a device
  * failure returns its status (tokens then hold the last good state).
- *   block_stats  host [n_blocks] or NULL: per block {steps, drafted, re-masked}
- *                (entries before first_block untouched)
+ *   block_stats  host [n_blocks] or NULL: per block {steps, drafted, re-masked,
+ *                drafted by the at-least-one rule} (entries before first_block
+ *                untouched; the last count needs flags and flags_host)
+ *   flags_host   host [n_seq, blk_len] or NULL: with flags, each step's flags
+ *                are copied here and the at-least-one drafts counted
  *   next_step    host or NULL: the global index after the last step run;
  *                with the block that follows, the point to resume from
  * counts, flags (optional), ws and ws_bytes are as for wino_step.
  */
 typedef const uint16_t *(*wino_hidden_fn)(void *user, int32_t step, int32_t blk_start);
 typedef struct {
-    int32_t steps, drafted, remasked;
+    int32_t steps, drafted, remasked, fallback;
 } wino_block_stats;
 WINO_API int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
                          int32_t n_blocks, int32_t first_block, int32_t first_step, wino_hidden_fn hidden,
-                         void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, void *ws,
-                         size_t ws_bytes, void *stream, wino_block_stats *block_stats, int32_t *next_step);
+                         void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, int8_t *flags_host,
+                         void *ws, size_t ws_bytes, void *stream, wino_block_stats *block_stats,
+                         int32_t *next_step);
 
 /*
  * Waits for `stream`, then reads the workspace status word written by the

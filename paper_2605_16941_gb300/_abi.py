@@ -53,7 +53,7 @@ class WinoParams(C.Structure):
 
 
 class WinoBlockStats(C.Structure):
-    _fields_ = [("steps", C.c_int32), ("drafted", C.c_int32), ("remasked", C.c_int32)]
+    _fields_ = [("steps", C.c_int32), ("drafted", C.c_int32), ("remasked", C.c_int32), ("fallback", C.c_int32)]
 
 
 # const uint16_t *(*)(void *user, int32_t step, int32_t blk_start)
@@ -98,7 +98,7 @@ def lib() -> C.CDLL:
         L.wino_version.argtypes = []
         L.wino_decode.restype = C.c_int
         L.wino_decode.argtypes = [vp, i64, i64, vp, C.POINTER(WinoParams), C.c_int32, C.c_int32, C.c_int32,
-                                  HIDDEN_FN, vp, vp, vp, vp, vp, sz, vp, C.POINTER(WinoBlockStats),
+                                  HIDDEN_FN, vp, vp, vp, vp, vp, vp, sz, vp, C.POINTER(WinoBlockStats),
                                   C.POINTER(C.c_int32)]
         _lib = L
     return _lib
@@ -206,11 +206,13 @@ def wino_step_static_scratch(H, W, tokens, params: WinoParams, counts, flags=Non
 
 
 def wino_decode(W, tokens, params: WinoParams, n_blocks: int, hidden, counts, counts_host, ws, flags=None,
-                stream=None, *, first_block: int = 0, first_step: int = 0, d: int | None = None,
+                stream=None, *, flags_host=None, first_block: int = 0, first_step: int = 0, d: int | None = None,
                 V: int | None = None):
     """The library's decode loop (wino_decode).  ``hidden(k, blk_start)`` returns step k's device bf16
     hidden states (a tensor, kept alive until the next call); ``counts_host`` is a host int32 [n_seq, 3]
-    tensor (pinned for speed).  Returns (status, per-block stats list, next step index); the status is
+    tensor (pinned for speed); with ``flags`` and a host int8 ``flags_host`` the at-least-one drafts are
+    counted too.  Returns (status, per-block (steps, drafted, re-masked, at-least-one drafts), next step
+    index); the status is
     WINO_OK or the error that stopped the loop (an exception raised by ``hidden`` is re-raised)."""
     d = int(W.shape[1]) if d is None else d
     V = int(W.shape[0]) if V is None else V
@@ -230,11 +232,12 @@ def wino_decode(W, tokens, params: WinoParams, n_blocks: int, hidden, counts, co
     nxt = C.c_int32(0)
     ws_bytes = ws.numel() * ws.element_size()
     rc = lib().wino_decode(_ptr(W), d, V, _ptr(tokens), C.byref(params), n_blocks, first_block, first_step, fn,
-                           None, _ptr(counts), _ptr(counts_host), _ptr(flags), _ptr(ws), ws_bytes, _stream(stream),
+                           None, _ptr(counts), _ptr(counts_host), _ptr(flags), _ptr(flags_host), _ptr(ws), ws_bytes,
+                           _stream(stream),
                            stats, C.byref(nxt))
     if failure:
         raise failure[0]
-    return rc, [(b.steps, b.drafted, b.remasked) for b in stats], nxt.value
+    return rc, [(b.steps, b.drafted, b.remasked, b.fallback) for b in stats], nxt.value
 
 
 def wino_read_device_status(ws, stream=None) -> int:

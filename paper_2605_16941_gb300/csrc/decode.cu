@@ -14,11 +14,12 @@
 
 extern "C" int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
                            int32_t n_blocks, int32_t first_block, int32_t first_step, wino_hidden_fn hidden,
-                           void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, void *ws,
-                           size_t ws_bytes, void *stream, wino_block_stats *block_stats, int32_t *next_step)
+                           void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, int8_t *flags_host,
+                           void *ws, size_t ws_bytes, void *stream, wino_block_stats *block_stats,
+                           int32_t *next_step)
 {
     const wino::Range range("wino_decode");
-    if (!W || !tokens || !p || !hidden || !counts || !counts_host || !ws)
+    if (!W || !tokens || !p || !hidden || !counts || !counts_host || !ws || (flags_host && !flags))
         return WINO_ERR_ARG;
     if (n_blocks < 1 || first_block < 0 || first_block > n_blocks || first_step < 0 || p->max_steps < 1)
         return WINO_ERR_ARG;
@@ -27,12 +28,13 @@ extern "C" int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tok
         return WINO_ERR_SHAPE;  // every block must lie inside the sequence
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const size_t count_bytes = (size_t)p->n_seq * 3 * sizeof(int32_t);
+    const size_t flag_bytes = (size_t)p->n_seq * p->blk_len;
     wino_params q = *p;
     int32_t k = first_step;
     int rc = WINO_OK;
     for (int32_t b = first_block; b < n_blocks && rc == WINO_OK; ++b) {
         q.blk_start = p->blk_start + b * p->blk_len;
-        wino_block_stats bs{0, 0, 0};
+        wino_block_stats bs{0, 0, 0, 0};
         for (;;) {
             if (bs.steps >= p->max_steps) {
                 rc = WINO_ERR_MAX_STEPS;
@@ -48,6 +50,7 @@ extern "C" int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tok
             if (rc != WINO_OK)
                 break;
             if (cudaMemcpyAsync(counts_host, counts, count_bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+                (flags_host && cudaMemcpyAsync(flags_host, flags, flag_bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess) ||
                 cudaStreamSynchronize(s) != cudaSuccess) {
                 rc = WINO_ERR_CUDA;
                 break;
@@ -65,6 +68,9 @@ extern "C" int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tok
             }
             if (rc != WINO_OK)
                 break;
+            if (flags_host)
+                for (size_t i = 0; i < flag_bytes; ++i)
+                    bs.fallback += (flags_host[i] == 2);  // drafted by the at-least-one rule
             ++k;
             ++bs.steps;
             if (done)

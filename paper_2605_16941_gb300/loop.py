@@ -27,7 +27,7 @@ class BlockStats:
     steps: int = 0
     drafted: int = 0
     remasked: int = 0
-    fallback_steps: int = 0  # steps on which some sequence drafted by the at-least-one rule only
+    fallback: int = 0  # drafts made by the at-least-one rule (no masked position cleared tau1)
 
 
 @dataclass
@@ -86,6 +86,7 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
     counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
+    flags_host = torch.zeros((n_seq, blk_len), dtype=torch.int8, pin_memory=True)
     tokens_host = torch.zeros((n_seq, S), dtype=torch.int32, pin_memory=True) if trajectory is not None else None
     if trajectory is not None:
         with torch.cuda.stream(ts):
@@ -107,6 +108,7 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
             wino_step(H, W, tokens, p, counts, ws, flags=flags, stream=ts)
             with torch.cuda.stream(ts):
                 counts_host.copy_(counts, non_blocking=True)
+                flags_host.copy_(flags, non_blocking=True)
                 if tokens_host is not None:
                     tokens_host.copy_(tokens, non_blocking=True)
             ts.synchronize()
@@ -118,6 +120,7 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
             bs.steps += 1
             bs.drafted += int(c[:, 0].sum())
             bs.remasked += int(c[:, 1].sum())
+            bs.fallback += int((flags_host.numpy() == 2).sum())
             stats.rows_scored += N
             if on_step is not None:
                 on_step(k, b0, c.copy(), flags)
@@ -149,16 +152,18 @@ def decode_native(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, ta
     ws = torch.zeros(wino_workspace_size_step(p, d, V), dtype=torch.uint8, device=dev)
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
+    flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
+    flags_host = torch.zeros((n_seq, blk_len), dtype=torch.int8, pin_memory=True)
     torch.cuda.current_stream(dev).synchronize()  # the buffers above are ready before the library's stream runs
-    rc, blocks, nxt = wino_decode(W, tokens, p, n_blocks, hidden, counts, counts_host, ws, stream=ts,
-                                  first_block=start_block, first_step=start_step)
+    rc, blocks, nxt = wino_decode(W, tokens, p, n_blocks, hidden, counts, counts_host, ws, flags=flags,
+                                  flags_host=flags_host, stream=ts, first_block=start_block, first_step=start_step)
     if rc != WINO_OK:
         raise WinoError(rc, f"wino_decode (stopped at step {nxt})")
     stats = LoopStats()
     for b in range(start_block, n_blocks):
-        steps, drafted, remasked = blocks[b]
+        steps, drafted, remasked, fallback = blocks[b]
         stats.blocks.append(BlockStats(block=b, blk_start=prompt_len + b * blk_len, steps=steps, drafted=drafted,
-                                       remasked=remasked))
+                                       remasked=remasked, fallback=fallback))
     stats.total_steps = nxt - start_step
     stats.rows_scored = N * stats.total_steps
     stats.next_step = nxt

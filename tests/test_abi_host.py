@@ -151,11 +151,11 @@ def test_decode_argument_errors():
     host = (C.c_int32 * 6)()
 
     def call(p, n_blocks=2, first_block=0, first_step=0, hidden=fn, **kw):
-        a = dict(W=FAKE, tok=FAKE, cnt=FAKE, cnth=C.addressof(host), ws=FAKE)
+        a = dict(W=FAKE, tok=FAKE, cnt=FAKE, cnth=C.addressof(host), fl=None, flh=None, ws=FAKE)
         a.update(kw)
         return L.wino_decode(a["W"], 64, 100, a["tok"], C.byref(p) if p is not None else None, n_blocks,
-                             first_block, first_step, hidden, None, a["cnt"], a["cnth"], None, a["ws"], 1 << 30,
-                             None, None, None)
+                             first_block, first_step, hidden, None, a["cnt"], a["cnth"], a["fl"], a["flh"], a["ws"],
+                             1 << 30, None, None, None)
     for k in ("W", "tok", "cnt", "cnth", "ws"):
         assert call(_p(), **{k: None}) == wino.WINO_ERR_ARG, k
     assert call(None) == wino.WINO_ERR_ARG
@@ -165,4 +165,5 @@ def test_decode_argument_errors():
     assert call(_p(), first_step=-1) == wino.WINO_ERR_ARG
     assert call(_p(max_steps=0)) == wino.WINO_ERR_ARG
     assert call(_p(), n_blocks=3) == wino.WINO_ERR_SHAPE  # blocks 32..80 run past seq_len 64
+    assert call(_p(), flh=C.addressof(host)) == wino.WINO_ERR_ARG  # host flags without device flags
     assert called == []

@@ -46,11 +46,11 @@ def test_native_loop_matches_python_loop(mode):
     tok_c, last_c = dev(st.tokens), torch.zeros_like(dev(st.tokens))
     got = loop.decode_native(Wd, tok_c, hidden=hidden, last_change=last_c, **_kw(w, **extra))
     assert np.array_equal(host(tok_c), host(tok_py)) and np.array_equal(host(last_c), host(last_py))
-    assert [(b.steps, b.drafted, b.remasked) for b in got.blocks] == [(b.steps, b.drafted, b.remasked)
-                                                                      for b in ref.blocks]
+    assert [(b.steps, b.drafted, b.remasked, b.fallback) for b in got.blocks] == \
+        [(b.steps, b.drafted, b.remasked, b.fallback) for b in ref.blocks]
     assert got.total_steps == ref.total_steps == got.next_step and got.rows_scored == ref.rows_scored
     assert not np.any(host(tok_c)[:, w.prompt_len:] == w.mask_id)
-    print(mode, [b.steps for b in got.blocks])
+    print(mode, [b.steps for b in got.blocks], "at-least-one drafts", [b.fallback for b in got.blocks])
 
 
 def test_native_loop_resumes_a_python_checkpoint():
