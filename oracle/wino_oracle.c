@@ -188,7 +188,7 @@ int oracle_row_targets(const int32_t *tokens, int64_t n_seq, int64_t seq_len, in
  * simultaneous.  counts[s] = {drafted (MASK -> token), re-masked, MASKs left
  * in the block}; flags[s * blk_len + l] (optional) gets the outcome codes.
  * With freeze_finished != 0, a sequence whose block has no MASK is not
- * stepped at all: the loop "until no MASK is left" (Sec. 4.2.3) has ended
+ * stepped at all: its loop, which runs until the block has no MASK (Sec. 4.2.3), has ended
  * for it.  If last_change (int32 [n_seq, seq_len]) is given, every position
  * whose token this step changes is set to step_index.
  *
