@@ -582,3 +582,56 @@ def test_decode_loop_checkpoint_resume():
         rest = loop.decode(Wd, tok_c, last_change=last_c, start_block=start_block, start_step=start_step, **kw)
         assert np.array_equal(host(tok_c), host(tok_a)) and np.array_equal(host(last_c), host(last_a)), stop_at
         assert start_step + rest.total_steps == full.total_steps and rest.next_step == full.next_step
+
+
+@pytest.mark.parametrize("name,mode", [("llada_b8", "compact"), ("unified_b4", "compact"), ("llada_b1", "no_shadow"),
+                                       ("llada_b8", "no_shadow"), ("llada_b8", "fixed_m4"),
+                                       ("unified_b4", "fixed_m4_verify")])
+def test_step_modes_full_size(name, mode):
+    """The step's other modes at the benchmark configurations' full sizes: row compaction gives the full
+    step's result; WINO+ and fixed-M steps equal the oracle's Eq. 4 on the GPU's own statistics, whose
+    sampled rows match the oracle's."""
+    import dataclasses
+
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import compare_rows, dev, f32, gpu_score, host
+    w = ws.WORKLOADS[name]
+    no_shadow = mode in ("no_shadow", "fixed_m4")
+    draft_m = 4 if mode.startswith("fixed_m4") else 0
+    if no_shadow:
+        w = dataclasses.replace(w, shadow=False)
+    W = ws.weights(w)
+    Wd = dev(W)
+    st = ws.initial_state(w)
+    H = ws.hidden_states(w, W, st, step=0)
+
+    def step(**opts):
+        tok_d = dev(st.tokens)
+        counts = torch.full((w.n_seq, 3), -9, dtype=torch.int32, device="cuda")
+        flags = torch.full((w.n_seq, w.blk_len), -9, dtype=torch.int8, device="cuda")
+        p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len, **opts)
+        wsp = wino.step_workspace(p, w.d, w.V)
+        wino.wino_step(dev(H), Wd, tok_d, p, counts, wsp, flags=flags)
+        torch.cuda.synchronize()
+        assert wino.wino_read_device_status(wsp) == wino.WINO_OK
+        return host(tok_d), host(counts), host(flags)
+
+    if mode == "compact":
+        full = step()
+        comp = step(compact=True)
+        assert all(np.array_equal(a, b) for a, b in zip(full, comp))
+        print(f"{name} compact: drafted {int(comp[1][:, 0].sum())} remasked {int(comp[1][:, 1].sum())}")
+        return
+    tok, cnt, fl = step(no_shadow=no_shadow, draft_m=draft_m)
+    t = None if no_shadow else oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
+    g = gpu_score(dev(H), Wd, t)
+    ref = oracle.draft_verify(st.tokens, st.blk_start, w.blk_len, w.mask_id, f32(w.tau1), f32(w.tau2), g.argmax,
+                              g.pmax.astype(np.float64), None if no_shadow else g.ptarget.astype(np.float64),
+                              no_shadow=no_shadow, draft_m=draft_m)
+    assert np.array_equal(tok, ref[0]) and np.array_equal(cnt, ref[1]) and np.array_equal(fl, ref[2])
+    rows = np.random.default_rng(5).choice(w.N, 16, replace=False)
+    rep = compare_rows(oracle.score_rows(H[rows], W, None if t is None else t[rows]), g, rows)
+    if draft_m:
+        masked = (st.tokens[:, st.blk_start:st.blk_start + w.blk_len] == w.mask_id).sum(1)
+        assert np.array_equal(((fl == 5) | (fl == 4)).sum(1), np.minimum(masked, draft_m))
+    print(f"{name} {mode}: {rep} drafted {int(cnt[:, 0].sum())} remasked {int(cnt[:, 1].sum())}")
