@@ -33,3 +33,29 @@ def test_bounded_wait_times_out_and_context_survives():
     torch.cuda.synchronize()
     assert wino.wino_read_device_status(wsp) == wino.WINO_OK
     assert np.all(host(counts) >= 0)
+
+
+def test_loop_driver_reports_a_device_failure(monkeypatch):
+    """A step whose bounded device wait expired reports WINO_ERR_DEVICE_TIMEOUT in every counts entry; the
+    decode loop stops there and raises it.  The failing step is a host-side fake (no GPU fault)."""
+    import paper_2605_16941_gb300 as wino
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import dev
+    w = ws.WORKLOADS["tiny"]
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    real_step = loop.wino_step
+    calls = []
+
+    def flaky_step(H, Wt, tokens, p, counts, wsp, flags=None, stream=None):
+        calls.append(p.step_index)
+        if len(calls) < 3:
+            return real_step(H, Wt, tokens, p, counts, wsp, flags=flags, stream=stream)
+        counts.fill_(wino.WINO_ERR_DEVICE_TIMEOUT)  # what the finish kernel writes after a timeout
+
+    monkeypatch.setattr(loop, "wino_step", flaky_step)
+    with pytest.raises(wino.WinoError) as e:
+        loop.decode(dev(W), dev(st.tokens), prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks,
+                     tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id,
+                     hidden=lambda k, b0: dev(ws.hidden_states(w, W, st, step=k)))
+    assert e.value.status == wino.WINO_ERR_DEVICE_TIMEOUT and calls == [1, 2, 3]
