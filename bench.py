@@ -529,7 +529,8 @@ def run_loop(args):
         tok = to_dev(st.tokens)
         stats = driver(Wd, tok, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks,
                        tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, max_steps=4096,
-                       compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m)
+                       compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m,
+                       skip_finished=args.skip_finished)
         return stats, tok
 
     t_gen = time.time()
@@ -558,6 +559,7 @@ def run_loop(args):
                  "remasked_per_block": [b.remasked for b in stats.blocks],
                  "fallback_drafts_per_block": [b.fallback for b in stats.blocks],
                  "total_steps": stats.total_steps, "repeats": len(runs),
+                 "rows_scored": stats.rows_scored, "rows_all_sequences": rows,
                  "timing": "wall clock around the whole decode (median of the repeats); hidden states resident "
                            "in device memory; includes the per-step counts read-back the loop needs",
                  "driver": "Python loop (loop.decode)" if args.python_loop else "library loop (wino_decode)"},
@@ -569,6 +571,9 @@ def run_loop(args):
         line["config"]["no_shadow"] = "WINO+ inference (WINO_OPT_NO_SHADOW): block rows only"
     if args.draft_m:
         line["config"]["draft_m"] = args.draft_m
+    if args.skip_finished:
+        line["config"]["skip_finished"] = ("only sequences whose block still has a MASK are scored (%d of %d rows); "
+                                           "value counts all sequences' rows" % (stats.rows_scored, rows))
     print(json.dumps(line), flush=True)
 
 
@@ -592,6 +597,8 @@ def main():
     ap.add_argument("--loop", action="store_true",
                     help="time the workload's whole decode loop (until no MASK is left) instead of K steps")
     ap.add_argument("--loop-repeats", type=int, default=3)
+    ap.add_argument("--skip-finished", action="store_true",
+                    help="with --loop: score only the sequences whose block still has a MASK")
     ap.add_argument("--python-loop", action="store_true",
                     help="with --loop: step from the Python driver (loop.decode) instead of the library's loop")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)

@@ -90,6 +90,15 @@ typedef struct {
                           tau1 is not used; M = 1 is high-confidence greedy decoding (Eq. 1).
                           Verification is unchanged; combine with WINO_OPT_NO_SHADOW for the
                           irreversible baseline decoders.  Must be >= 0. */
+    const int32_t *active_seq; /* optional device int32 [n_active] (wino_step only): the sequences this
+                          step scores and updates, each in [0, n_seq), no repeats.  H keeps its full
+                          layout for all n_seq sequences; the step gathers the listed sequences' rows
+                          (with WINO_OPT_COMPACT only the row each position reads) into the workspace
+                          and scores those alone; every other sequence's tokens, counts and flags are
+                          left as they are.  A batched decode lists the sequences whose block still
+                          has a MASK: the others' loops have ended (as WINO_OPT_FREEZE_FINISHED), so
+                          their rows need not be scored.  NULL: every sequence. */
+    int32_t n_active;  /* entries of active_seq, 1..n_seq, when active_seq is not NULL */
 } wino_params;
 
 /*
@@ -133,9 +142,11 @@ typedef struct {
 WINO_API int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes);
 
 /*
- * Workspace bytes wino_step needs for these parameters (row layout and
- * WINO_OPT_COMPACT taken into account); >= wino_workspace_size of the rows it
- * scores.
+ * Workspace bytes wino_step needs for these parameters (row layout,
+ * WINO_OPT_COMPACT and an active-sequence list taken into account); >=
+ * wino_workspace_size of the rows it scores.  With active_seq set, the size
+ * depends on n_active only: a workspace sized for n_active = n_seq serves
+ * every list.
  */
 WINO_API int wino_workspace_size_step(const wino_params *p, int64_t d, int64_t V, size_t *bytes);
 
@@ -175,7 +186,8 @@ WINO_API int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, in
  *          (the position stays MASK and is not counted as drafted),
  *          5 drafted by the fixed-M rule (draft_m > 0)
  * Ties in the at-least-one rule go to the smallest position.  Requires
- * 0 <= tau1, tau2 <= 1, 1 <= blk_len <= 1024, n_seq >= 1, draft_m >= 0.
+ * 0 <= tau1, tau2 <= 1, 1 <= blk_len <= 1024, n_seq >= 1, draft_m >= 0 and
+ * active_seq == NULL (the rows are the caller's).
  */
 WINO_API int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream);
@@ -238,9 +250,16 @@ WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int6
  * decodes want WINO_OPT_FREEZE_FINISHED.  A block that is still not done
  * after p->max_steps (>= 1) steps returns WINO_ERR_MAX_STEPS; a device
  * failure returns its status (tokens then hold the last good state).
+ *   active_buf   device int32 [n_seq] or NULL: when given, every step lists in
+ *                it the sequences whose current block still has a MASK and
+ *                scores only those (see wino_params.active_seq; p->active_seq
+ *                itself must be NULL); ws must then be sized for n_active =
+ *                n_seq.  With WINO_OPT_FREEZE_FINISHED (which it implies for the
+ *                sequences it leaves out) the same states as without it.
  *   block_stats  host [n_blocks] or NULL: per block {steps, drafted, re-masked,
- *                drafted by the at-least-one rule} (entries before first_block
- *                untouched; the last count needs flags and flags_host)
+ *                drafted by the at-least-one rule, sequences stepped summed
+ *                over the steps} (entries before first_block untouched; the
+ *                at-least-one count needs flags and flags_host)
  *   flags_host   host [n_seq, blk_len] or NULL: with flags, each step's flags
  *                are copied here and the at-least-one drafts counted
  *   next_step    host or NULL: the global index after the last step run;
@@ -250,12 +269,13 @@ WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int6
 typedef const uint16_t *(*wino_hidden_fn)(void *user, int32_t step, int32_t blk_start);
 typedef struct {
     int32_t steps, drafted, remasked, fallback;
+    int32_t seq_steps; /* sequences stepped, summed over the block's steps */
 } wino_block_stats;
 WINO_API int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *tokens, const wino_params *p,
                          int32_t n_blocks, int32_t first_block, int32_t first_step, wino_hidden_fn hidden,
                          void *user, int32_t *counts, int32_t *counts_host, int8_t *flags, int8_t *flags_host,
-                         void *ws, size_t ws_bytes, void *stream, wino_block_stats *block_stats,
-                         int32_t *next_step);
+                         int32_t *active_buf, void *ws, size_t ws_bytes, void *stream,
+                         wino_block_stats *block_stats, int32_t *next_step);
 
 /*
  * Waits for `stream`, then reads the workspace status word written by the

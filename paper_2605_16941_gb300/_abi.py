@@ -49,11 +49,13 @@ class WinoParams(C.Structure):
     _fields_ = [("tau1", C.c_float), ("tau2", C.c_float), ("mask_id", C.c_int32), ("n_seq", C.c_int32),
                 ("seq_len", C.c_int32), ("blk_start", C.c_int32), ("blk_len", C.c_int32),
                 ("max_steps", C.c_int32), ("options", C.c_int32), ("step_index", C.c_int32),
-                ("last_change", C.c_void_p), ("draft_m", C.c_int32)]
+                ("last_change", C.c_void_p), ("draft_m", C.c_int32), ("active_seq", C.c_void_p),
+                ("n_active", C.c_int32)]
 
 
 class WinoBlockStats(C.Structure):
-    _fields_ = [("steps", C.c_int32), ("drafted", C.c_int32), ("remasked", C.c_int32), ("fallback", C.c_int32)]
+    _fields_ = [("steps", C.c_int32), ("drafted", C.c_int32), ("remasked", C.c_int32), ("fallback", C.c_int32),
+                ("seq_steps", C.c_int32)]
 
 
 # const uint16_t *(*)(void *user, int32_t step, int32_t blk_start)
@@ -98,7 +100,7 @@ def lib() -> C.CDLL:
         L.wino_version.argtypes = []
         L.wino_decode.restype = C.c_int
         L.wino_decode.argtypes = [vp, i64, i64, vp, C.POINTER(WinoParams), C.c_int32, C.c_int32, C.c_int32,
-                                  HIDDEN_FN, vp, vp, vp, vp, vp, vp, sz, vp, C.POINTER(WinoBlockStats),
+                                  HIDDEN_FN, vp, vp, vp, vp, vp, vp, vp, sz, vp, C.POINTER(WinoBlockStats),
                                   C.POINTER(C.c_int32)]
         _lib = L
     return _lib
@@ -160,12 +162,16 @@ def workspace(N: int, d: int, V: int, device=None):
 
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
                 max_steps: int = 4096, freeze_finished: bool = False, step_index: int = 0,
-                last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0) -> WinoParams:
-    """wino_params; ``draft_m`` > 0 selects fixed-M drafting (naive parallel sampling, Sec. 3)."""
+                last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0,
+                active_seq=None, n_active: int | None = None) -> WinoParams:
+    """wino_params; ``draft_m`` > 0 selects fixed-M drafting (naive parallel sampling, Sec. 3);
+    ``active_seq`` (device int32) lists the sequences a wino_step scores and updates (default: all)."""
     opts = ((WINO_OPT_FREEZE_FINISHED if freeze_finished else 0) | (WINO_OPT_NO_SHADOW if no_shadow else 0) |
             (WINO_OPT_COMPACT if compact else 0))
+    if active_seq is not None and n_active is None:
+        n_active = int(active_seq.numel())
     return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps, opts, step_index,
-                      _ptr(last_change), draft_m)
+                      _ptr(last_change), draft_m, _ptr(active_seq), n_active or 0)
 
 
 def wino_score_rows(H, W, target, argmax, pmax, ptarget, ws, stream=None, *, entropy=None, N: int | None = None,
@@ -206,13 +212,14 @@ def wino_step_static_scratch(H, W, tokens, params: WinoParams, counts, flags=Non
 
 
 def wino_decode(W, tokens, params: WinoParams, n_blocks: int, hidden, counts, counts_host, ws, flags=None,
-                stream=None, *, flags_host=None, first_block: int = 0, first_step: int = 0, d: int | None = None,
-                V: int | None = None):
+                stream=None, *, flags_host=None, active_buf=None, first_block: int = 0, first_step: int = 0,
+                d: int | None = None, V: int | None = None):
     """The library's decode loop (wino_decode).  ``hidden(k, blk_start)`` returns step k's device bf16
     hidden states (a tensor, kept alive until the next call); ``counts_host`` is a host int32 [n_seq, 3]
     tensor (pinned for speed); with ``flags`` and a host int8 ``flags_host`` the at-least-one drafts are
-    counted too.  Returns (status, per-block (steps, drafted, re-masked, at-least-one drafts), next step
-    index); the status is
+    counted too; with a device int32 [n_seq] ``active_buf`` only the sequences whose block still has a
+    MASK are stepped.  Returns (status, per-block (steps, drafted, re-masked, at-least-one drafts,
+    sequences stepped summed over the steps), next step index); the status is
     WINO_OK or the error that stopped the loop (an exception raised by ``hidden`` is re-raised)."""
     d = int(W.shape[1]) if d is None else d
     V = int(W.shape[0]) if V is None else V
@@ -232,12 +239,12 @@ def wino_decode(W, tokens, params: WinoParams, n_blocks: int, hidden, counts, co
     nxt = C.c_int32(0)
     ws_bytes = ws.numel() * ws.element_size()
     rc = lib().wino_decode(_ptr(W), d, V, _ptr(tokens), C.byref(params), n_blocks, first_block, first_step, fn,
-                           None, _ptr(counts), _ptr(counts_host), _ptr(flags), _ptr(flags_host), _ptr(ws), ws_bytes,
-                           _stream(stream),
+                           None, _ptr(counts), _ptr(counts_host), _ptr(flags), _ptr(flags_host), _ptr(active_buf),
+                           _ptr(ws), ws_bytes, _stream(stream),
                            stats, C.byref(nxt))
     if failure:
         raise failure[0]
-    return rc, [(b.steps, b.drafted, b.remasked, b.fallback) for b in stats], nxt.value
+    return rc, [(b.steps, b.drafted, b.remasked, b.fallback, b.seq_steps) for b in stats], nxt.value
 
 
 def wino_read_device_status(ws, stream=None) -> int:

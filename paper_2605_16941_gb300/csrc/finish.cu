@@ -84,11 +84,13 @@ struct Eq4Smem {
     float conf[kMaxBlkLen];  // fixed-M drafting: pmax of each masked position, -inf elsewhere
 };
 
-// Eq. 4 on sequence s by the whole CTA (kFinishRows warps; thread t owns positions t, t + 256, ...).
-// Every load is issued before any decision so the update costs about one memory round trip.
-// Statistics are read through L2: other CTAs of the same launch may have written them.
-__device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
-                          const wino_params &p, int32_t *counts, int8_t *flags, int32_t status, Eq4Smem &sm)
+// Eq. 4 on sequence s by the whole CTA (kFinishRows warps; thread t owns positions t, t + 256, ...),
+// reading the statistics of the a-th sequence of the scored rows (a = s unless an active-sequence list
+// chose the rows).  Every load is issued before any decision so the update costs about one memory round
+// trip.  Statistics are read through L2: other CTAs of the same launch may have written them.
+__device__ void eq4_block(int a, int s, int32_t *tokens, const int32_t *argmax, const float *pmax,
+                          const float *ptarget, const wino_params &p, int32_t *counts, int8_t *flags, int32_t status,
+                          Eq4Smem &sm)
 {
     constexpr int kT = kFinishRows * 32;
     constexpr int kPer = kMaxBlkLen / kT;
@@ -103,8 +105,8 @@ __device__ void eq4_block(int s, int32_t *tokens, const int32_t *argmax, const f
     const bool shadow = !(p.options & WINO_OPT_NO_SHADOW);  // WINO+ inference has no verification rows
     const bool compact = (p.options & WINO_OPT_COMPACT) != 0;  // one row per position
     int32_t *y = tokens + (int64_t)s * p.seq_len + p.blk_start;
-    const int64_t rb = (int64_t)((shadow && !compact) ? 2 * s : s) * L;  // rows read for masked positions
-    const int64_t rs = (int64_t)(compact ? s : 2 * s + 1) * L;         // rows read for decoded positions
+    const int64_t rb = (int64_t)((shadow && !compact) ? 2 * a : a) * L;  // rows read for masked positions
+    const int64_t rs = (int64_t)(compact ? a : 2 * a + 1) * L;         // rows read for decoded positions
 
     int32_t yv[kPer], av[kPer];
     float pm[kPer], pt[kPer];
@@ -354,8 +356,15 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
     }
     __syncthreads();
     const int nd = s_ndone;
-    for (int i = 0; i < nd; ++i)
-        eq4_block(s_done[i], a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status, sm);
+    for (int i = 0; i < nd; ++i) {
+        const int sq = a.p.active_seq ? a.p.active_seq[s_done[i]] : s_done[i];
+        if (sq < 0 || sq >= a.p.n_seq) {  // a bad entry of the caller's list: no update, an error status
+            if (threadIdx.x == 0 && a.status)
+                atomicExch(a.status, (int32_t)WINO_ERR_ARG);
+            continue;
+        }
+        eq4_block(s_done[i], sq, a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status, sm);
+    }
 }
 
 // Eq. 4 alone, one CTA per sequence.
@@ -364,7 +373,7 @@ __global__ void __launch_bounds__(kFinishRows * 32)
                         const wino_params p, int32_t *counts, int8_t *flags)
 {
     __shared__ Eq4Smem sm;
-    eq4_block(blockIdx.x, tokens, argmax, pmax, ptarget, p, counts, flags, WINO_OK, sm);
+    eq4_block(blockIdx.x, blockIdx.x, tokens, argmax, pmax, ptarget, p, counts, flags, WINO_OK, sm);
 }
 
 // Row compaction: one CTA per position copies the one row Eq. 4 will read -- the block row of a masked
@@ -384,6 +393,44 @@ __global__ void __launch_bounds__(256) gather_compact_kernel(const uint4 *__rest
         dst[i] = __ldg(src + i);
 }
 
+// Active-sequence gather: one CTA per scored row copies the row of a listed sequence (row r of the
+// gathered layout belongs to the a-th listed sequence s) into the workspace with 16-byte loads, and
+// writes the row's target: the current token of the position a shadow row verifies, else -1 (MASK or
+// a block row), so that the score kernel reads the gathered rows with explicit targets.
+__global__ void __launch_bounds__(256) gather_active_kernel(const uint4 *__restrict__ H, uint4 *__restrict__ Hc,
+                                                            int32_t *__restrict__ target,
+                                                            const int32_t *__restrict__ tokens, const wino_params p,
+                                                            int64_t vec_per_row)
+{
+    ptx::grid_dep_wait();  // the token state may still be being written by the previous step
+    ptx::grid_dep_launch_dependents();
+    const bool shadow = !(p.options & WINO_OPT_NO_SHADOW);
+    const bool compact = (p.options & WINO_OPT_COMPACT) != 0;
+    const int64_t L = p.blk_len;
+    const int64_t per_seq = (shadow && !compact) ? 2 * L : L;
+    const int64_t r = blockIdx.x;
+    const int64_t a = r / per_seq, j = r - a * per_seq;
+    const int64_t s = p.active_seq[a];
+    uint4 *dst = Hc + r * vec_per_row;
+    if (s < 0 || s >= p.n_seq) {  // a bad entry of the caller's list: read nothing (the finish kernel reports it)
+        for (int64_t i = threadIdx.x; i < vec_per_row; i += blockDim.x)
+            dst[i] = make_uint4(0, 0, 0, 0);
+        if (threadIdx.x == 0)
+            target[r] = -1;
+        return;
+    }
+    const int64_t l = (j < L) ? j : j - L;
+    const int32_t y = tokens[s * p.seq_len + p.blk_start + l];
+    // kind of the row: the shadow row for j >= L; with compaction, the row Eq. 4 reads for this position
+    const int kind = !shadow ? 0 : (compact ? (y == p.mask_id ? 0 : 1) : (j < L ? 0 : 1));
+    const int64_t src_row = shadow ? (2 * s + kind) * L + l : s * L + l;
+    const uint4 *src = H + src_row * vec_per_row;
+    for (int64_t i = threadIdx.x; i < vec_per_row; i += blockDim.x)
+        dst[i] = __ldg(src + i);
+    if (threadIdx.x == 0)
+        target[r] = (kind == 1 && y != p.mask_id) ? y : -1;
+}
+
 }  // namespace
 
 cudaError_t launch_gather_compact(const uint16_t *H, uint16_t *Hc, const int32_t *tokens, const wino_params &p,
@@ -400,6 +447,22 @@ cudaError_t launch_gather_compact(const uint16_t *H, uint16_t *Hc, const int32_t
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, gather_compact_kernel, reinterpret_cast<const uint4 *>(H),
                               reinterpret_cast<uint4 *>(Hc), tokens, p, d / 8);
+}
+
+cudaError_t launch_gather_active(const uint16_t *H, uint16_t *Hc, int32_t *target, const int32_t *tokens,
+                                 const wino_params &p, int64_t rows, int64_t d, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)rows);
+    cfg.blockDim = dim3(256);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gather_active_kernel, reinterpret_cast<const uint4 *>(H),
+                              reinterpret_cast<uint4 *>(Hc), target, tokens, p, d / 8);
 }
 
 cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream)

@@ -92,7 +92,7 @@ struct FinishArgs {
     float *entropy;       // optional: H(p) = -sum_v p_v log p_v per row
     int32_t G, N, V;
     TargetSource ts;
-    const int32_t *status;
+    int32_t *status;  // read; set to WINO_ERR_ARG when an active-sequence list entry is out of range
     int32_t *argmax;
     float *pmax;
     float *ptarget;
@@ -116,6 +116,8 @@ cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const S
 cudaError_t launch_finish(const FinishArgs &a, cudaStream_t stream);
 
 // Row compaction (WINO_OPT_COMPACT): Hc[s*L + l] = H[(2s + (tokens[s, b0 + l] == MASK ? 0 : 1)) * L + l].
+cudaError_t launch_gather_active(const uint16_t *H, uint16_t *Hc, int32_t *target, const int32_t *tokens,
+                                 const wino_params &p, int64_t rows, int64_t d, cudaStream_t stream);
 cudaError_t launch_gather_compact(const uint16_t *H, uint16_t *Hc, const int32_t *tokens, const wino_params &p,
                                   int64_t d, cudaStream_t stream);
 

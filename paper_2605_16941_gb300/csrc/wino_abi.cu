@@ -181,8 +181,10 @@ int check_params(const wino_params *p)
         return WINO_ERR_ARG;
     if (!(p->tau1 >= 0.f && p->tau1 <= 1.f) || !(p->tau2 >= 0.f && p->tau2 <= 1.f) || p->draft_m < 0)
         return WINO_ERR_ARG;
-    if (!aligned(p->last_change, 4))
+    if (!aligned(p->last_change, 4) || !aligned(p->active_seq, 4))
         return WINO_ERR_ARG;
+    if (p->active_seq && (p->n_active < 1 || p->n_active > p->n_seq))
+        return WINO_ERR_SHAPE;
     if (p->n_seq < 1 || p->blk_len < 1 || p->blk_len > kMaxBlkLen || p->blk_start < 0 || p->seq_len < 1 ||
         (int64_t)p->blk_start + p->blk_len > p->seq_len || p->mask_id < 0)
         return WINO_ERR_SHAPE;
@@ -261,15 +263,17 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
 int64_t step_rows(const wino_params &p)
 {
     const bool one_row = (p.options & (WINO_OPT_NO_SHADOW | WINO_OPT_COMPACT)) != 0;
-    return (int64_t)p.n_seq * (one_row ? 1 : 2) * p.blk_len;
+    return (int64_t)(p.active_seq ? p.n_active : p.n_seq) * (one_row ? 1 : 2) * p.blk_len;
 }
 
 size_t step_ws_bytes(const wino_params &p, int64_t d, int64_t V)
 {
     const int64_t rows = step_rows(p);
     size_t total = ws_layout(rows, V).total;
-    if (p.options & WINO_OPT_COMPACT)
+    if ((p.options & WINO_OPT_COMPACT) || p.active_seq)
         total += round_up((size_t)rows * (size_t)d * 2, kAlign);  // the gathered rows
+    if (p.active_seq)
+        total += round_up((size_t)rows * 4, kAlign);  // and their targets
     return total;
 }
 
@@ -341,7 +345,8 @@ int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax,
                       const wino_params *p, int32_t *counts, int8_t *flags, void *stream)
 {
     const Range range("wino_draft_verify");
-    if (!tokens || !argmax || !pmax || !counts || !p || (!ptarget && !(p->options & WINO_OPT_NO_SHADOW)))
+    if (!tokens || !argmax || !pmax || !counts || !p || (!ptarget && !(p->options & WINO_OPT_NO_SHADOW)) ||
+        p->active_seq)
         return WINO_ERR_ARG;
     if (!aligned(tokens, 4) || !aligned(argmax, 4) || !aligned(pmax, 4) || !aligned(ptarget, 4) ||
         !aligned(counts, 4))
@@ -392,6 +397,19 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     ts.compact = compact ? 1 : 0;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const uint16_t *Hs = H;
+    if (p->active_seq) {  // gather the listed sequences' rows (and their targets) behind the workspace proper
+        DeviceInfo info;
+        if ((rc = device_info(&info)) != WINO_OK)
+            return rc;
+        uint16_t *Hc = reinterpret_cast<uint16_t *>(w8 + L.total);
+        int32_t *tgt = reinterpret_cast<int32_t *>(w8 + L.total + round_up((size_t)N * (size_t)d * 2, kAlign));
+        if (launch_gather_active(H, Hc, tgt, tokens, *p, N, d, s) != cudaSuccess)
+            return WINO_ERR_CUDA;
+        TargetSource tsa{};
+        tsa.target = tgt;
+        return score_and_finish(Hc, W, N, d, V, tsa, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s,
+                                true);
+    }
     if (compact) {  // gather the one row per position Eq. 4 reads, behind the workspace proper
         DeviceInfo info;
         if ((rc = device_info(&info)) != WINO_OK)

@@ -53,7 +53,7 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
            hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
            on_step: Callable | None = None, last_change=None, no_shadow: bool = False,
            compact: bool = False, draft_m: int = 0, trajectory: list | None = None, start_block: int = 0,
-           start_step: int = 0) -> LoopStats:
+           start_step: int = 0, skip_finished: bool = False) -> LoopStats:
     """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
 
     ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
@@ -72,16 +72,22 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     states (Sec. 5.1-5.2); it costs one extra device-to-host copy of ``tokens`` per step.
     ``start_block``, ``start_step``: resume a checkpointed decode (see ``resume_point``): blocks
     before ``start_block`` are taken as done and the global step count starts at ``start_step``.
+    ``skip_finished``: each step scores only the sequences whose block still has a MASK (an
+    active-sequence list, ``wino_params.active_seq``); the states are those of the frozen
+    sequences without it, and ``on_step`` sees zero counts for the sequences left out.
     """
+    import numpy as np
     import torch
 
     n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
     d, V = int(W.shape[1]), int(W.shape[0])
-    N = n_seq * (1 if (no_shadow or compact) else 2) * blk_len  # rows scored per step
+    rows_per_seq = (1 if (no_shadow or compact) else 2) * blk_len  # rows scored per sequence and step
     dev = tokens.device
     ts = stream if stream is not None else torch.cuda.current_stream(dev)  # every copy goes on the step's stream
+    active_d = torch.arange(n_seq, dtype=torch.int32, device=dev) if skip_finished else None
+    active_h = torch.zeros(n_seq, dtype=torch.int32, pin_memory=True) if skip_finished else None
     p0 = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact,
-                     draft_m=draft_m)
+                     draft_m=draft_m, active_seq=active_d, n_active=n_seq if skip_finished else None)
     ws = torch.zeros(wino_workspace_size_step(p0, d, V), dtype=torch.uint8, device=dev)
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
@@ -100,11 +106,17 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
         p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True,
                         last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
         bs = BlockStats(block=b, blk_start=b0)
+        active = list(range(n_seq))  # a new block: every sequence takes part
         while True:
             if bs.steps >= max_steps:
                 raise WinoError(WINO_ERR_MAX_STEPS, f"decode: block {b} not finished after {max_steps} steps")
             H = hidden(k, b0)
             p.step_index = k + 1
+            if skip_finished:
+                active_h[:len(active)] = torch.tensor(active, dtype=torch.int32)
+                with torch.cuda.stream(ts):
+                    active_d[:len(active)].copy_(active_h[:len(active)], non_blocking=True)
+                p.active_seq, p.n_active = active_d.data_ptr(), len(active)
             wino_step(H, W, tokens, p, counts, ws, flags=flags, stream=ts)
             with torch.cuda.stream(ts):
                 counts_host.copy_(counts, non_blocking=True)
@@ -112,7 +124,13 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
                 if tokens_host is not None:
                     tokens_host.copy_(tokens, non_blocking=True)
             ts.synchronize()
-            c = counts_host.numpy()
+            c = counts_host.numpy().copy()
+            fl = flags_host.numpy().copy()
+            if skip_finished:  # the sequences left out were not stepped: no counts, no flags
+                left_out = np.ones(n_seq, bool)
+                left_out[active] = False
+                c[left_out] = 0
+                fl[left_out] = 0
             if tokens_host is not None:
                 trajectory.append(tokens_host.numpy().copy())
             if (c < 0).any():
@@ -120,13 +138,15 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
             bs.steps += 1
             bs.drafted += int(c[:, 0].sum())
             bs.remasked += int(c[:, 1].sum())
-            bs.fallback += int((flags_host.numpy() == 2).sum())
-            stats.rows_scored += N
+            bs.fallback += int((fl == 2).sum())
+            stats.rows_scored += rows_per_seq * len(active)
             if on_step is not None:
                 on_step(k, b0, c.copy(), flags)
             k += 1
             if (c[:, 2] == 0).all():
                 break
+            if skip_finished:
+                active = [i for i in active if c[i, 2] != 0]
         stats.blocks.append(bs)
     stats.total_steps = k - start_step
     stats.next_step = k
@@ -136,35 +156,40 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
 def decode_native(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float,
                   mask_id: int, hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
                   last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0,
-                  start_block: int = 0, start_step: int = 0) -> LoopStats:
+                  start_block: int = 0, start_step: int = 0, skip_finished: bool = False) -> LoopStats:
     """``decode`` with the step loop run by the library (``wino_decode``): the same steps, states and
     statistics, with one callback into Python per step (for the hidden states) instead of the whole
-    per-step bookkeeping.  No ``on_step`` or ``trajectory``; errors raise ``WinoError``."""
+    per-step bookkeeping.  No ``on_step`` or ``trajectory``; errors raise ``WinoError``.
+    ``skip_finished`` as in ``decode``: the library keeps the active-sequence list."""
     import torch
 
     n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
     d, V = int(W.shape[1]), int(W.shape[0])
-    N = n_seq * (1 if (no_shadow or compact) else 2) * blk_len
+    rows_per_seq = (1 if (no_shadow or compact) else 2) * blk_len
     dev = tokens.device
     ts = stream if stream is not None else torch.cuda.current_stream(dev)
     p = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, max_steps, freeze_finished=True,
                     last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
-    ws = torch.zeros(wino_workspace_size_step(p, d, V), dtype=torch.uint8, device=dev)
+    active_buf = torch.zeros(n_seq, dtype=torch.int32, device=dev) if skip_finished else None
+    p_ws = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact,
+                       active_seq=active_buf, n_active=n_seq if skip_finished else None)  # sized for every list
+    ws = torch.zeros(wino_workspace_size_step(p_ws, d, V), dtype=torch.uint8, device=dev)
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     counts_host = torch.zeros((n_seq, 3), dtype=torch.int32, pin_memory=True)
     flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
     flags_host = torch.zeros((n_seq, blk_len), dtype=torch.int8, pin_memory=True)
     torch.cuda.current_stream(dev).synchronize()  # the buffers above are ready before the library's stream runs
     rc, blocks, nxt = wino_decode(W, tokens, p, n_blocks, hidden, counts, counts_host, ws, flags=flags,
-                                  flags_host=flags_host, stream=ts, first_block=start_block, first_step=start_step)
+                                  flags_host=flags_host, active_buf=active_buf, stream=ts, first_block=start_block,
+                                  first_step=start_step)
     if rc != WINO_OK:
         raise WinoError(rc, f"wino_decode (stopped at step {nxt})")
     stats = LoopStats()
     for b in range(start_block, n_blocks):
-        steps, drafted, remasked, fallback = blocks[b]
+        steps, drafted, remasked, fallback, seq_steps = blocks[b]
         stats.blocks.append(BlockStats(block=b, blk_start=prompt_len + b * blk_len, steps=steps, drafted=drafted,
                                        remasked=remasked, fallback=fallback))
+        stats.rows_scored += rows_per_seq * seq_steps
     stats.total_steps = nxt - start_step
-    stats.rows_scored = N * stats.total_steps
     stats.next_step = nxt
     return stats

@@ -102,6 +102,7 @@ def test_draft_verify_argument_errors():
     assert call(_p(n_seq=0)) == wino.WINO_ERR_SHAPE
     assert call(_p(mask_id=-1)) == wino.WINO_ERR_SHAPE
     assert call(_p(draft_m=-1)) == wino.WINO_ERR_ARG
+    assert call(_p(active_seq=FAKE, n_active=1)) == wino.WINO_ERR_ARG  # the caller's rows: no list
     for k in ("tok", "am", "pm", "pt", "cnt"):
         assert call(_p(), **{k: FAKE + 2}) == wino.WINO_ERR_ARG, k
     assert call(_p(last_change=FAKE + 3)) == wino.WINO_ERR_ARG
@@ -122,6 +123,9 @@ def test_step_argument_errors():
     assert call(_p(), tok=FAKE + 2) == wino.WINO_ERR_ARG
     assert call(_p(), cnt=FAKE + 1) == wino.WINO_ERR_ARG
     assert call(_p(last_change=FAKE + 2)) == wino.WINO_ERR_ARG
+    assert call(_p(active_seq=FAKE + 2, n_active=1)) == wino.WINO_ERR_ARG  # misaligned list
+    assert call(_p(active_seq=FAKE, n_active=0)) == wino.WINO_ERR_SHAPE
+    assert call(_p(active_seq=FAKE, n_active=3)) == wino.WINO_ERR_SHAPE  # more entries than sequences (2)
 
 
 def test_params_layout_matches_header(tmp_path):
@@ -151,11 +155,11 @@ def test_decode_argument_errors():
     host = (C.c_int32 * 6)()
 
     def call(p, n_blocks=2, first_block=0, first_step=0, hidden=fn, **kw):
-        a = dict(W=FAKE, tok=FAKE, cnt=FAKE, cnth=C.addressof(host), fl=None, flh=None, ws=FAKE)
+        a = dict(W=FAKE, tok=FAKE, cnt=FAKE, cnth=C.addressof(host), fl=None, flh=None, act=None, ws=FAKE)
         a.update(kw)
         return L.wino_decode(a["W"], 64, 100, a["tok"], C.byref(p) if p is not None else None, n_blocks,
-                             first_block, first_step, hidden, None, a["cnt"], a["cnth"], a["fl"], a["flh"], a["ws"],
-                             1 << 30, None, None, None)
+                             first_block, first_step, hidden, None, a["cnt"], a["cnth"], a["fl"], a["flh"], a["act"],
+                             a["ws"], 1 << 30, None, None, None)
     for k in ("W", "tok", "cnt", "cnth", "ws"):
         assert call(_p(), **{k: None}) == wino.WINO_ERR_ARG, k
     assert call(None) == wino.WINO_ERR_ARG
@@ -166,4 +170,5 @@ def test_decode_argument_errors():
     assert call(_p(max_steps=0)) == wino.WINO_ERR_ARG
     assert call(_p(), n_blocks=3) == wino.WINO_ERR_SHAPE  # blocks 32..80 run past seq_len 64
     assert call(_p(), flh=C.addressof(host)) == wino.WINO_ERR_ARG  # host flags without device flags
+    assert call(_p(active_seq=FAKE, n_active=1)) == wino.WINO_ERR_ARG  # the loop keeps its own list
     assert called == []

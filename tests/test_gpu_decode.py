@@ -6,6 +6,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import wino_synth as ws
 
 pytestmark = pytest.mark.gpu
@@ -114,3 +115,88 @@ def test_native_loop_errors():
     torch.cuda.synchronize()
     assert (host(ref)[:, w.prompt_len:w.prompt_len + w.blk_len] == w.mask_id).any(), "block 0 needs two steps"
     assert np.array_equal(host(tok1), host(ref))
+
+
+@pytest.mark.parametrize("mode", ["wino", "compact", "wino_plus"])
+def test_step_with_an_active_list(mode):
+    """A step over a list of sequences (unordered) scores and updates those alone: their results match the
+    oracle's step on just those sequences; every other sequence's tokens, counts and flags stay as they were."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import compare_step, dev, host
+    base = ws.Workload("active", d=256, V=5000, n_seq=6, blk_len=32, bias=((1.0, 0.0, 10.0),), predecoded=0.5)
+    w = ws.coverage_variant(base)
+    if mode == "wino_plus":
+        w = dataclasses.replace(w, shadow=False)
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    H = ws.hidden_states(w, W, st, step=1)
+    listed = [4, 1, 3]
+    act = dev(np.array(listed, np.int32))
+    opts = {"wino": {}, "compact": {"compact": True}, "wino_plus": {"no_shadow": True}}[mode]
+    p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len, active_seq=act,
+                         **opts)
+    tok_d = dev(st.tokens)
+    counts = torch.full((w.n_seq, 3), -9, dtype=torch.int32, device="cuda")
+    flags = torch.full((w.n_seq, w.blk_len), -9, dtype=torch.int8, device="cuda")
+    wsp = wino.step_workspace(p, w.d, w.V)
+    wino.wino_step(dev(H), dev(W), tok_d, p, counts, wsp, flags=flags)
+    torch.cuda.synchronize()
+    assert wino.wino_read_device_status(wsp) == wino.WINO_OK
+    tok, cnt, fl = host(tok_d), host(counts), host(flags)
+    others = [s for s in range(w.n_seq) if s not in listed]
+    assert np.array_equal(tok[others], st.tokens[others])
+    assert np.all(cnt[others] == -9) and np.all(fl[others] == -9)
+    # the oracle's step on the listed sequences alone (rows of each listed sequence, in list order)
+    rows_per_seq = w.kinds * w.blk_len
+    H_sub = np.concatenate([H[s * rows_per_seq:(s + 1) * rows_per_seq] for s in listed])
+    o = oracle.step(H_sub, W, st.tokens[listed], st.blk_start, w.blk_len, w.mask_id, w.tau1, w.tau2,
+                    no_shadow=(mode == "wino_plus"))
+    if mode == "wino_plus":  # compare_step reads the [s][kind][l] layout: give it block rows twice
+        o = dataclasses.replace(o)
+        o.pmax = np.repeat(o.pmax.reshape(len(listed), 1, w.blk_len), 2, axis=1).reshape(-1)
+        o.gap = np.repeat(o.gap.reshape(len(listed), 1, w.blk_len), 2, axis=1).reshape(-1)
+        o.ptarget = np.ones(2 * len(listed) * w.blk_len)
+    rep = compare_step(st.tokens[listed], tok[listed], cnt[listed], o, st.blk_start, w.blk_len, w.mask_id, w.tau1,
+                       w.tau2)
+    print(mode, rep)
+
+
+def test_step_active_list_with_a_bad_entry():
+    """An out-of-range entry of the list is caught by the kernels' own checks: nothing is read or written for
+    it, the valid entries are stepped, and the device status reports WINO_ERR_ARG."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, host
+    w = ws.coverage_variant(ws.WORKLOADS["tiny"])
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    H = ws.hidden_states(w, W, st, step=0)
+    act7 = dev(np.array([7], np.int32))  # n_seq is 1: entry 7 is out of range
+    p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len, active_seq=act7)
+    tok_d = dev(st.tokens)
+    counts = torch.full((w.n_seq, 3), -9, dtype=torch.int32, device="cuda")
+    wsp = wino.step_workspace(p, w.d, w.V)
+    wino.wino_step(dev(H), dev(W), tok_d, p, counts, wsp)
+    torch.cuda.synchronize()
+    assert wino.wino_read_device_status(wsp) == wino.WINO_ERR_ARG
+    assert np.array_equal(host(tok_d), st.tokens) and np.all(host(counts) == -9)
+
+
+@pytest.mark.parametrize("native", [False, True], ids=["python", "library"])
+def test_decode_skipping_finished_sequences(native):
+    """Skipping the sequences whose block is done reaches the same states, finalization steps and per-block
+    counts as stepping every sequence (frozen), while scoring fewer rows."""
+    import paper_2605_16941_gb300.loop as loop
+    from gpu_helpers import dev, host
+    w = ws.Workload("skip_loop", d=64, V=1000, n_seq=6, blk_len=8, bias=((1.0, 1.0, 6.0),), n_blocks=3,
+                    bias_step=0.4, tau1=0.7, tau2=0.9)
+    Wd, st, hidden = _setup(w)
+    tok_a, last_a = dev(st.tokens), torch.zeros_like(dev(st.tokens))
+    ref = loop.decode(Wd, tok_a, hidden=hidden, last_change=last_a, **_kw(w))
+    drive = loop.decode_native if native else loop.decode
+    tok_b, last_b = dev(st.tokens), torch.zeros_like(dev(st.tokens))
+    got = drive(Wd, tok_b, hidden=hidden, last_change=last_b, skip_finished=True, **_kw(w))
+    assert np.array_equal(host(tok_b), host(tok_a)) and np.array_equal(host(last_b), host(last_a))
+    assert [(b.steps, b.drafted, b.remasked, b.fallback) for b in got.blocks] == \
+        [(b.steps, b.drafted, b.remasked, b.fallback) for b in ref.blocks]
+    assert got.rows_scored < ref.rows_scored
+    print("rows scored", got.rows_scored, "of", ref.rows_scored)
