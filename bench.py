@@ -1,22 +1,26 @@
 #!/usr/bin/env python3
 """Throughput of one WINO step (fused LM head + vocabulary softmax + Eq. 4 revoke) on GB300.
 
-Workload: the LLaDA-8B-shaped single step (d=4096, V=126464, one sequence,
-block of 128 plus 128 shadow rows: N=256 scored rows), seeded synthetic
-inputs (wino_synth).  A step is one wino_step call through the C ABI: the
-fused score kernel (LM-head GEMM + online vocabulary softmax on 2-SM tensor
-core tiles) and the finish kernel (cross-tile merge + Eq. 4 update).
+Workload (default): the unified text+image vocabulary step, the largest of the
+single-GPU configurations: d=4096, V=134400, 4 sequences of a 256-position block
+plus its 256 shadow rows (N=2048 scored rows), seeded synthetic inputs
+(wino_synth).  A step is one wino_step call through the C ABI: the fused score
+kernel (LM-head GEMM + online vocabulary softmax on 2-SM tensor-core tiles) and
+the finish kernel (cross-tile merge + Eq. 4 update).
 
 Prints one JSON line (rank 0).  `value` is scored rows/s over the K timed
-steps with inputs resident in HBM (W is 1.04 GB, larger than L2, so no L2
+steps with inputs resident in HBM (W is 1.1 GB, larger than L2, so no L2
 flush is needed); `e2e` is the same metric with each step's hidden states
 and token state copied in from pinned host memory and the tokens and counts
 copied back, through the same C ABI; `roofline` rates the dominant kernel
 (the fused score kernel, timed by CUDA events the library records around
 each launch on the launch stream, in a second region of K steps) against the
-measured HBM copy bandwidth;
-`cpu_baseline` times the fp64 CPU oracle on a bounded sample of the same
-workload on this host's cores.
+measured peak of its bound; `configs` repeats the step and kernel timing, at
+the same K, on the three LLaDA-8B-shaped configurations (one sequence, N=256;
+eight sequences, N=2048; the 16-sequence decode step, N=1024); `cpu_baseline`
+times the fp64 CPU oracle on a bounded sample of the workload's rows on this
+host's cores, and `parity` compares one whole GPU step with the oracle's whole
+step (every row scored in fp64).
 
 --impl reference times the oracle itself as the reference arm (CPU, fp64).
 Multi-GPU (torchrun): every rank decodes its own replica (weak scaling); no
@@ -161,6 +165,165 @@ def gpu_uuid(dev):
         return s if s.startswith("GPU-") else "GPU-" + s
     except Exception:
         return None
+
+
+def roofline_terms(w, rows_scored, peaks):
+    """Algorithmic work of one score launch (2 N d V flops; W and H read once, 12 B of results per row) and
+    the time each would take at the measured peaks."""
+    flops = 2.0 * rows_scored * w.d * w.V
+    w_bytes = w.V * w.d * 2.0
+    alg_bytes = w_bytes + rows_scored * w.d * 2.0 + 12.0 * rows_scored
+    t_flop = flops / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = alg_bytes / (peaks["hbm_gbs"] * 1e9)
+    return flops, w_bytes, alg_bytes, t_flop, t_hbm, ("hbm" if t_hbm >= t_flop else "tensor")
+
+
+def kernel_roofline(w, rows_scored, peaks, score_avg_s):
+    """The score kernel's achieved rate against the measured peak of its bound."""
+    flops, w_bytes, alg_bytes, t_flop, t_hbm, bound = roofline_terms(w, rows_scored, peaks)
+    if bound == "hbm":
+        achieved, peak, unit = alg_bytes / score_avg_s / 1e9, peaks["hbm_gbs"], "GB/s"
+    else:
+        achieved, peak, unit = flops / score_avg_s / 1e12, peaks["bf16_tflops"], "TFLOP/s"
+    tflops = flops / score_avg_s / 1e12
+    return {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+            "algorithmic_per_launch": {"bytes": alg_bytes, "flops": flops}, "avg_launch_us": score_avg_s * 1e6,
+            "tensor_tflops": tflops, "tensor_frac": tflops / peaks["bf16_tflops"],
+            "tensor_frac_sustained": tflops / peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])}
+
+
+def time_steps(step, steps, stream, dev):
+    """K calls of step(i) back to back between two CUDA events on the launch stream (ms)."""
+    import torch
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    ev0.record(stream)
+    for i in range(steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    return ev0.elapsed_time(ev1)
+
+
+def time_score_kernel(wino, step, steps, dev):
+    """Average duration (s) of the score kernel over K more steps, from the CUDA events the library records
+    around each of its launches on the launch stream (this serialises the launches)."""
+    import torch
+    torch.cuda.synchronize(dev)
+    wino.wino_profile_begin(steps)
+    for i in range(steps):
+        step(i)
+    score_ms, score_n = wino.wino_profile_end()
+    torch.cuda.synchronize(dev)
+    return (score_ms / max(1, score_n)) / 1e3, score_n
+
+
+def measure_configs(names, args, wino, ws, dev, sid, peaks, to_dev):
+    """Step and score-kernel timing of other configurations at the same step count (resident inputs)."""
+    import torch
+    out, w_cache = {}, {}
+    for name in names:
+        w = ws.WORKLOADS[name]
+        key = (w.d, w.V, w.seed)
+        if key not in w_cache:
+            w_cache.clear()  # one extra LM head resident at a time
+            W = ws.weights(w)
+            w_cache[key] = (W, to_dev(W))
+        W, Wd = w_cache[key]
+        st = ws.initial_state(w)
+        Hd = [to_dev(ws.hidden_states(w, W, st, step=k)) for k in range(2)]
+        tok = to_dev(st.tokens)
+        counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device=dev)
+        wsp = wino.workspace(w.N, w.d, w.V, device=dev)
+        p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len)
+
+        def step(i):
+            wino.wino_step(Hd[i % 2], Wd, tok, p, counts, wsp, stream=sid)
+
+        for i in range(args.warmup):
+            step(i)
+        ms = time_steps(step, args.steps, torch.cuda.current_stream(dev), dev)
+        score_avg_s, _ = time_score_kernel(wino, step, args.steps, dev)
+        if wino.wino_read_device_status(wsp, stream=sid) != wino.WINO_OK:
+            raise RuntimeError(f"device status not OK on {name}")
+        flops, w_bytes, _, t_flop, _, _ = roofline_terms(w, w.N, peaks)
+        step_s = ms / 1e3 / args.steps
+        out[name] = {"workload": w.name, "N": w.N, "d": w.d, "V": w.V, "steps": args.steps,
+                     "ms_per_step": ms / args.steps, "rows_per_s": w.N / step_s,
+                     "tflops_per_step": flops / step_s / 1e12,
+                     "step_roofline_frac": max(t_flop, w_bytes / (peaks["hbm_gbs"] * 1e9)) / step_s,
+                     "kernel_roofline": kernel_roofline(w, w.N, peaks, score_avg_s)}
+        del Hd, tok, wsp
+    return out
+
+
+def oracle_baseline_and_parity(w, W, H, st, gpu_stats, tok_gpu, cnt_gpu, budget_s: float = 15.0):
+    """The fp64 oracle on every row of one step of the workload.  A first chunk of rows (about budget_s of
+    CPU work) is the timed CPU baseline; all rows then give the oracle's whole step, compared with one GPU
+    step from the same state: per-row probabilities within 1e-3, argmax and token state exact outside the
+    counted near-tie and near-threshold positions (the tolerances of the parity tests)."""
+    import numpy as np
+
+    import oracle
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    from gpu_helpers import PROB_TOL, TIE_TOL, flagged_positions
+    nt = oracle.num_threads()
+    t = oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
+    n1 = min(nt, w.N)
+    t0 = time.perf_counter()
+    first = oracle.score_rows(H[:n1], W, t[:n1])
+    t_first = time.perf_counter() - t0
+    chunk = int(min(w.N - n1, max(nt, nt * round(budget_s / t_first))))
+    parts = [first]
+    t_chunk = t_rest = 0.0
+    if chunk > 0:
+        t0 = time.perf_counter()
+        parts.append(oracle.score_rows(H[n1:n1 + chunk], W, t[n1:n1 + chunk]))
+        t_chunk = time.perf_counter() - t0
+    timed_rows, timed_s = (chunk, t_chunk) if chunk > 0 else (n1, t_first)
+    cpu = {"value": timed_rows / timed_s, "unit": UNIT, "cores": nt, "kind": "oracle",
+           "sample": f"{timed_rows} of the {w.N} rows of one step of {w.name}, each scored over the full vocabulary "
+                     f"in fp64 ({timed_s:.1f} s); the Eq. 4 update (microseconds) is not included",
+           "seconds": timed_s}
+    if n1 + chunk < w.N:
+        t0 = time.perf_counter()
+        parts.append(oracle.score_rows(H[n1 + chunk:], W, t[n1 + chunk:]))
+        t_rest = time.perf_counter() - t0
+    o = type(first)(*(np.concatenate([getattr(x, f) for x in parts]) for f in first.__dataclass_fields__))
+    tok, cnt, fl = oracle.draft_verify(st.tokens, st.blk_start, w.blk_len, w.mask_id, w.tau1, w.tau2, o.argmax,
+                                       o.pmax, o.ptarget)
+    ostep = oracle.StepResult(tok, cnt, fl, o.argmax, o.pmax, o.ptarget, o.gap)
+    flag = flagged_positions(st.tokens, ostep, st.blk_start, w.blk_len, w.mask_id, w.tau1, w.tau2)
+    b0, L = st.blk_start, w.blk_len
+    g_blk, o_blk = tok_gpu[:, b0:b0 + L], tok[:, b0:b0 + L]
+    outside = np.ones(st.tokens.shape[1], bool)
+    outside[b0:b0 + L] = False
+    near = o.gap < TIE_TOL
+    clean = ~flag.any(1)
+    parity = {
+        "rows": int(w.N), "oracle": "fp64 CPU oracle, every row over the full vocabulary, then Eq. 4",
+        "tolerance": f"per-row probabilities within {PROB_TOL} absolute; argmax and token state exact except at "
+                     f"positions whose top-2 logits differ by < {TIE_TOL} or whose decision probability lies within "
+                     f"{PROB_TOL} of its threshold (flagged, counted)",
+        "max_abs_dpmax": float(np.abs(gpu_stats.pmax.astype(np.float64) - o.pmax).max()),
+        "max_abs_dptarget": float(np.abs(gpu_stats.ptarget.astype(np.float64) - o.ptarget).max()),
+        "argmax_mismatch_outside_near_ties": int(((gpu_stats.argmax != o.argmax) & ~near).sum()),
+        "argmax_near_ties": int(near.sum()),
+        "token_mismatch_outside_flagged": int(((g_blk != o_blk) & ~flag).sum()),
+        "flagged_positions": int(flag.sum()),
+        "flagged_mismatch": int(((g_blk != o_blk) & flag).sum()),
+        "positions_outside_block_changed": int((tok_gpu[:, outside] != st.tokens[:, outside]).sum()),
+        "counts_mismatch_unflagged_sequences": int((cnt_gpu[clean] != cnt[clean]).any(1).sum()),
+        "oracle_branches": {"threshold_drafts": int((fl == oracle.FLAG_DRAFT).sum()),
+                            "fallback_drafts": int((fl == oracle.FLAG_DRAFT_FALLBACK).sum()),
+                            "remasked": int((fl == oracle.FLAG_REMASK).sum())},
+        "oracle_seconds": t_first + t_chunk + t_rest,
+    }
+    parity["ok"] = (parity["max_abs_dpmax"] <= PROB_TOL and parity["max_abs_dptarget"] <= PROB_TOL and
+                    parity["argmax_mismatch_outside_near_ties"] == 0 and parity["token_mismatch_outside_flagged"] == 0
+                    and parity["positions_outside_block_changed"] == 0
+                    and parity["counts_mismatch_unflagged_sequences"] == 0)
+    return cpu, parity
 
 
 def oracle_cpu_baseline(w, W, H, targets, budget_s: float = 12.0, max_rows: int = 256):
@@ -421,30 +584,42 @@ def run_wino(args, rank, world, local_rank):
 
     peaks, peak_src = load_peaks()
     rows_scored = w.N // 2 if args.compact else w.N  # rows the score kernel actually multiplies
-    flops = 2.0 * rows_scored * w.d * w.V
-    w_bytes = w.V * w.d * 2.0
-    h_bytes = rows_scored * w.d * 2.0
-    alg_bytes = w_bytes + h_bytes + 12.0 * rows_scored
-    t_flop = flops / (peaks["bf16_tflops"] * 1e12)
-    t_hbm = alg_bytes / (peaks["hbm_gbs"] * 1e9)
-    bound = "hbm" if t_hbm >= t_flop else "tensor"
+    flops, w_bytes, alg_bytes, t_flop, t_hbm, bound = roofline_terms(w, rows_scored, peaks)
     score_avg_s = (score_ms / max(1, score_n)) / 1e3
-    if bound == "hbm":
-        achieved, peak, unit = alg_bytes / score_avg_s / 1e9, peaks["hbm_gbs"], "GB/s"
-    else:
-        achieved, peak, unit = flops / score_avg_s / 1e12, peaks["bf16_tflops"], "TFLOP/s"
+    roof = kernel_roofline(w, rows_scored, peaks, score_avg_s)
     step_s = t_max / 1e3 / args.steps
     value = job_rows_per_s(w.N, args.steps, world, t_max / 1e3)
     clock_info = clocks.summary(tw0, tw1) if clocks else None
 
-    cpu = None
+    # The other LLaDA-shaped configurations at the same step count (rank 0 only).
+    configs = None
+    plain = not (args.no_shadow or score_only or args.compact or args.draft_m or args.graph)
+    if plain and not args.no_configs:
+        names = [n for n in ("llada_b1", "llada_b8", "loop_b16") if n != args.workload]
+        configs = measure_configs(names, args, wino, ws, dev, sid, peaks, to_dev)
+
+    cpu, parity = None, None
     if world == 1 and not args.no_cpu_baseline:
         import oracle
-        if args.no_shadow or score_only:  # rows without a target
-            t = np.full(w.N, -1, np.int32)
+        if plain:
+            # one GPU step and the GPU's statistics of every row, from the initial state; then the oracle
+            tok1 = to_dev(st.tokens)
+            cnt1 = torch.zeros_like(counts)
+            ws1 = wino.workspace(w.N, w.d, w.V, device=dev)
+            wino.wino_step(Hd[0], Wd, tok1, p, cnt1, ws1, stream=sid)
+            t_rows = to_dev(oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id))
+            wino.wino_score_rows(Hd[0], Wd, t_rows, am, pm, pt, ws1, stream=sid)
+            torch.cuda.synchronize(dev)
+            if wino.wino_read_device_status(ws1, stream=sid) != wino.WINO_OK:
+                raise RuntimeError("device status not OK in the parity step")
+            from types import SimpleNamespace
+            g = SimpleNamespace(argmax=am.cpu().numpy(), pmax=pm.cpu().numpy(), ptarget=pt.cpu().numpy())
+            cpu, parity = oracle_baseline_and_parity(w, W, Hs[0], st, g, tok1.cpu().numpy(), cnt1.cpu().numpy(),
+                                                     budget_s=args.cpu_budget_s)
         else:
-            t = oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
-        cpu = oracle_cpu_baseline(w, W, Hs[0], t, budget_s=args.cpu_budget_s)
+            t = np.full(w.N, -1, np.int32) if (args.no_shadow or score_only) else \
+                oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id)
+            cpu = oracle_cpu_baseline(w, W, Hs[0], t, budget_s=args.cpu_budget_s)
 
     cfg = config_dict(w)
     if args.no_shadow:
@@ -462,15 +637,11 @@ def run_wino(args, rank, world, local_rank):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": cfg,
-        "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+        "roofline": {**{k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac")},
                      "traffic": ncu_traffic(w.name), "kernel": "score_kernel (fused LM-head GEMM + online vocab softmax)",
-                     "algorithmic_per_launch": {"bytes": alg_bytes, "flops": flops},
-                     "avg_launch_us": score_avg_s * 1e6, "launches_timed": score_n, "peak_source": peak_src,
-                     "timing": "per-launch CUDA events around the score kernel over a second region of K steps",
-                     "tensor_tflops": flops / score_avg_s / 1e12,
-                     "tensor_frac": flops / score_avg_s / 1e12 / peaks["bf16_tflops"],
-                     "tensor_frac_sustained": flops / score_avg_s / 1e12 / peaks.get("bf16_tflops_sustained",
-                                                                                      peaks["bf16_tflops"])},
+                     **{k: v for k, v in roof.items() if k not in ("bound", "achieved", "peak", "unit", "frac")},
+                     "launches_timed": score_n, "peak_source": peak_src,
+                     "timing": "per-launch CUDA events around the score kernel over a second region of K steps"},
         "step_roofline_frac": max(t_flop, w_bytes / (peaks["hbm_gbs"] * 1e9)) / step_s,
         "tflops_per_step": flops / step_s / 1e12,
         "e2e": None if not e2e_steps else {
@@ -479,6 +650,8 @@ def run_wino(args, rank, world, local_rank):
         "gpu_launches": (3 if args.compact and not score_only else 2) * args.steps,  # (gather +) score + finish
         "clocks": clock_info,
         "cpu_baseline": cpu,
+        "parity": parity,
+        "configs": configs,
     }
     print(json.dumps(line), flush=True)
     if world > 1:
@@ -583,8 +756,11 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["wino", "reference"], default="wino")
-    ap.add_argument("--workload", default="llada_b1")
-    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="unified_b4")
+    ap.add_argument("--no-cpu-baseline", action="store_true",
+                    help="skip the oracle legs (CPU baseline and whole-step parity)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the timing of the other LLaDA-shaped configurations")
     ap.add_argument("--compact", action="store_true",
                     help="row compaction: score only the row each position's update reads (not the headline: "
                          "the metric counts all 2*n_seq*blk_len rows)")
@@ -601,7 +777,7 @@ def main():
                     help="with --loop: score only the sequences whose block still has a MASK")
     ap.add_argument("--python-loop", action="store_true",
                     help="with --loop: step from the Python driver (loop.decode) instead of the library's loop")
-    ap.add_argument("--cpu-budget-s", type=float, default=12.0)
+    ap.add_argument("--cpu-budget-s", type=float, default=15.0)
     ap.add_argument("--ref-budget-s", type=float, default=90.0)
     args = ap.parse_args()
     if args.warmup < 3:

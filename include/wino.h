@@ -26,14 +26,14 @@
  *     current-block row of position l, kind 1 = its shadow-block row; row
  *     index n = (2*s + kind)*blk_len + l, N = 2*n_seq*blk_len.
  *   - `stream` is a cudaStream_t (NULL = legacy default stream); all work is
- *     enqueued on it asynchronously, in order.  Consecutive WINO calls on one
- *     stream overlap (programmatic dependent launch): a call may start reading
- *     its H and W while the previous WINO call's last kernel is finishing, so
- *     H and W must not be memory that the previous call writes (its tokens,
- *     counts, flags, statistics or workspace).
+ *     enqueued on it asynchronously, in order.  The kernels are launched with
+ *     programmatic dependent launch: a call's first kernel sets up (barriers,
+ *     tensor memory, L2 prefetches of its first H and W tiles) while the
+ *     kernel before it on the stream finishes, and reads nothing from global
+ *     memory until that kernel has completed, whatever it is.
  *   - Return value: WINO_OK (0) or a negative wino_status.  On an argument
  *     error nothing is enqueued.  Device-side failures (a bounded wait that
- *     expired) are reported in the workspace status word, see
+ *     expired) are reported through the workspace's status words, see
  *     wino_read_device_status.
  *   - Devices: compute capability 10.3 (GB300).  Other devices get
  *     WINO_ERR_UNSUPPORTED.
@@ -132,10 +132,14 @@ typedef struct {
 #define WINO_OPT_COMPACT 4
 
 /*
- * Bytes of scratch the score path needs for N rows of dimension d over a
- * vocabulary of V entries (per-tile partial softmax statistics, targets and
- * per-row results, plus one status word).  `ws` passed to wino_score_rows /
- * wino_step must hold at least this many bytes and be 256-byte aligned.
+ * Bytes of scratch wino_score_rows needs for N rows of dimension d over a
+ * vocabulary of V entries, with or without the entropy output: status words,
+ * per-sequence tickets, per-row partial softmax records (R = min(ceil(V/128),
+ * 256) of 16 bytes per row, plus R floats per row only used for the entropy)
+ * and the per-row results.  Without an entropy output the call needs R * 4 * N
+ * bytes (rounded to 256) less.  `ws` must be 256-byte aligned and zero-filled
+ * before its first use (for example with cudaMemsetAsync); the library keeps
+ * its status words consistent from then on, so a workspace is reused as it is.
  * Returns WINO_ERR_SHAPE for sizes the kernels do not support, see
  * wino_score_rows.
  */
@@ -143,10 +147,13 @@ WINO_API int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
 
 /*
  * Workspace bytes wino_step needs for these parameters (row layout,
- * WINO_OPT_COMPACT and an active-sequence list taken into account); >=
- * wino_workspace_size of the rows it scores.  With active_seq set, the size
- * depends on n_active only: a workspace sized for n_active = n_seq serves
- * every list.
+ * WINO_OPT_COMPACT and an active-sequence list taken into account): the
+ * scratch of wino_score_rows without entropy for the rows it scores, plus
+ * 2*d bytes per scored row for the gathered rows of WINO_OPT_COMPACT or an
+ * active-sequence list (and 4 bytes per row for their targets with a list).
+ * With active_seq set, the size depends on n_active only: a workspace sized
+ * for n_active = n_seq serves every list.  Zero-filled before first use, as
+ * for wino_workspace_size.
  */
 WINO_API int wino_workspace_size_step(const wino_params *p, int64_t d, int64_t V, size_t *bytes);
 
@@ -165,7 +172,8 @@ WINO_API int wino_workspace_size_step(const wino_params *p, int64_t d, int64_t V
  *           Eq. 6-7); NULL skips it (the decode path never computes it)
  * Shapes: 1 <= N <= 2^24, 8 <= d <= 65536 with d % 8 == 0, 2 <= V <= 2^27.
  * Logits are accumulated in fp32 on the tensor cores; the softmax runs in
- * fp32.  The status word in `ws` is cleared at the start of the call.
+ * fp32.  ws_bytes must be at least wino_workspace_size(N, d, V) with an
+ * entropy output and R * 4 * N bytes less without one (see there).
  */
 WINO_API int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V,
                     const int32_t *target, int32_t *argmax, float *pmax, float *ptarget, float *entropy,
@@ -216,16 +224,23 @@ WINO_API int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t 
  * Same arguments, kernels and results as wino_step, with the workspace taken
  * from one fixed array of WINO_STATIC_SCRATCH_BYTES in device memory that the
  * library reserves on every GPU that loads it, until the process exits.  The
- * call allocates nothing.  Problems whose wino_workspace_size exceeds the
- * array are rejected with WINO_ERR_WORKSPACE before anything is launched
- * (for V >= 32768, any d: N = 2 * n_seq * blk_len up to 3266 rows).
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress); make that first call before any stream capture.
- * Every call on a device shares the one array: calls that may overlap on the
- * GPU (different streams, or host threads without ordering) race and must be
- * serialised by the caller.  The kernels clear the words they rely on (status
- * word, tickets) at the start of each call, so the array needs no
- * initialisation; the per-row statistics it holds are not returned.
+ * call allocates nothing.  A problem is accepted iff
+ * wino_workspace_size_step(p, d, V) <= WINO_STATIC_SCRATCH_BYTES, and
+ * rejected otherwise with WINO_ERR_WORKSPACE before anything is launched.
+ * Each scored row needs R * 16 + 14 bytes, R = min(ceil(V/128), 256), so for
+ * V > 32640 (R = 256): up to 4080 scored rows (N = 2 * n_seq * blk_len,
+ * any d); with WINO_OPT_COMPACT or an active-sequence list the gathered rows
+ * add 2*d bytes per scored row: at d = 4096, up to 1363 scored rows
+ * (n_seq * blk_len with WINO_OPT_COMPACT).
+ * Every call looks up the array's device address with the device current
+ * (cudaGetSymbolAddress); the first call on a device also clears the status
+ * words at the start of the array on `stream` (cudaMemsetAsync), so make that
+ * first call before any stream capture.  Every call on a device shares the
+ * one array: calls that may overlap on the GPU (different streams, or host
+ * threads without ordering) race and must be serialised by the caller.  The
+ * array keeps the last call's contents; the kernels clear what they rely on
+ * (tickets, status words) as each call goes, and the per-row statistics it
+ * holds are not returned.
  */
 #define WINO_STATIC_SCRATCH_BYTES (16u << 20)
 WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_t *tokens,
@@ -278,8 +293,10 @@ WINO_API int wino_decode(const uint16_t *W, int64_t d, int64_t V, int32_t *token
                          wino_block_stats *block_stats, int32_t *next_step);
 
 /*
- * Waits for `stream`, then reads the workspace status word written by the
- * last score launch that used `ws`: WINO_OK, or WINO_ERR_DEVICE_TIMEOUT.
+ * Waits for `stream`, then reads the outcome of the last call that used `ws`
+ * (published by its last kernel): WINO_OK, WINO_ERR_DEVICE_TIMEOUT (a bounded
+ * wait expired), WINO_ERR_ARG (an active-sequence list entry out of range) or
+ * WINO_ERR_UNSUPPORTED (the TMEM allocation check failed).
  */
 WINO_API int wino_read_device_status(const void *ws, void *stream, int *device_status);
 
@@ -294,6 +311,33 @@ WINO_API int wino_read_device_status(const void *ws, void *stream, int *device_s
  */
 WINO_API int wino_profile_begin(int max_launches);
 WINO_API int wino_profile_end(double *score_ms_total, int *score_launches);
+
+/*
+ * Timeline of the score kernel (diagnostics; the paper has no counterpart).
+ * Between wino_timeline_begin and wino_timeline_end, score launch i (from
+ * wino_score_rows or wino_step, counted from begin) writes, per CTA c, eight
+ * 64-bit words at buf[((i % n_launches) * ctas_per_launch + c) * 8]:
+ * %globaltimer stamps in ns of [0] kernel entry, [1] set-up done (barriers,
+ * tensor memory), [2] first tensor copy issued, [3] wait for the previous
+ * kernel done, [4] last MMA completed (leader CTA of a pair) or last tile
+ * read (the other CTA), [5] all roles done, [6] exit; and [7] = SM id << 32
+ * | tiles of the CTA pair (leader CTA).  A launch with more CTAs than
+ * ctas_per_launch writes nothing.  buf is a device buffer of
+ * n_launches * ctas_per_launch * 8 uint64 owned by the caller; end returns how
+ * many launches were counted.  One timeline per process at a time.
+ */
+WINO_API int wino_timeline_begin(uint64_t *buf, int64_t n_launches, int64_t ctas_per_launch);
+WINO_API int wino_timeline_end(int64_t *launches);
+
+/*
+ * How a score launch of N rows over V entries is split on the current device
+ * (diagnostics; the paper has no counterpart): plan (host int32[6]) receives
+ * the tile width bn, the vocabulary tiles n_vt = ceil(V / bn), the 256-row
+ * blocks n_mb, the row-block groups, the CTA pairs per group G (= records per
+ * row) and the grid size in CTAs.  Pair c of the launch serves row blocks
+ * c % groups (+ groups, ...) and, within each, tiles c / groups (+ G, ...).
+ */
+WINO_API int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan);
 
 /*
  * Self-test of the failure path (device-side timeout handling; the paper has

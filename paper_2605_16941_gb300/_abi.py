@@ -24,7 +24,7 @@ WINO_ERR_DEVICE_TIMEOUT = -6
 WINO_ERR_UNSUPPORTED = -7
 
 # per-position outcome codes written to `flags`
-FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK = 0, 1, 2, 3, 4
+FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK, FLAG_DRAFT_TOP_M = 0, 1, 2, 3, 4, 5
 
 # wino_params.options
 WINO_OPT_FREEZE_FINISHED = 1
@@ -33,7 +33,11 @@ WINO_OPT_COMPACT = 4
 
 EXPORTS = ("wino_workspace_size", "wino_workspace_size_step", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
-           "wino_selftest_wait_timeout", "wino_status_string", "wino_version", "wino_decode")
+           "wino_selftest_wait_timeout", "wino_status_string", "wino_version", "wino_decode", "wino_timeline_begin",
+           "wino_timeline_end", "wino_score_plan")
+
+# 64-bit words per CTA in a score-kernel timeline (wino_timeline_begin)
+TIMELINE_WORDS = 8
 
 # size of the fixed device array behind wino_step_static_scratch
 WINO_STATIC_SCRATCH_BYTES = 16 << 20
@@ -92,6 +96,12 @@ def lib() -> C.CDLL:
         L.wino_profile_begin.argtypes = [C.c_int]
         L.wino_profile_end.restype = C.c_int
         L.wino_profile_end.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_int)]
+        L.wino_score_plan.restype = C.c_int
+        L.wino_score_plan.argtypes = [i64, i64, i64, C.POINTER(C.c_int32)]
+        L.wino_timeline_begin.restype = C.c_int
+        L.wino_timeline_begin.argtypes = [vp, i64, i64]
+        L.wino_timeline_end.restype = C.c_int
+        L.wino_timeline_end.argtypes = [C.POINTER(i64)]
         L.wino_selftest_wait_timeout.restype = C.c_int
         L.wino_selftest_wait_timeout.argtypes = [vp, i64, vp]
         L.wino_status_string.restype = C.c_char_p
@@ -262,6 +272,26 @@ def wino_profile_end() -> tuple[float, int]:
     ms, n = C.c_double(0), C.c_int(0)
     _check(lib().wino_profile_end(C.byref(ms), C.byref(n)), "wino_profile_end")
     return ms.value, n.value
+
+
+def wino_score_plan(N: int, d: int, V: int) -> dict:
+    """The score kernel's work split for N rows over V entries on the current device."""
+    out = (C.c_int32 * 6)()
+    _check(lib().wino_score_plan(int(N), int(d), int(V), out), "wino_score_plan")
+    return dict(zip(("bn", "n_vt", "n_mb", "n_groups", "G", "ctas"), list(out)))
+
+
+def wino_timeline_begin(buf, n_launches: int, ctas_per_launch: int) -> None:
+    """Start recording per-CTA score-kernel stamps into the device uint64 tensor ``buf``
+    (n_launches * ctas_per_launch * TIMELINE_WORDS words)."""
+    _check(lib().wino_timeline_begin(_ptr(buf), int(n_launches), int(ctas_per_launch)), "wino_timeline_begin")
+
+
+def wino_timeline_end() -> int:
+    """Stop recording; returns the number of score launches counted."""
+    n = C.c_int64(0)
+    _check(lib().wino_timeline_end(C.byref(n)), "wino_timeline_end")
+    return n.value
 
 
 def wino_selftest_wait_timeout(status, limit_ns: int, stream=None) -> None:

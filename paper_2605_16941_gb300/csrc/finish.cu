@@ -14,7 +14,9 @@
 // and update need one launch.  Tickets are cleared by the score kernel of the
 // same step.  The kernel is launched programmatically: its launch overlaps the
 // score kernel and it waits (griddepcontrol.wait) for the score kernel's
-// results before touching them.
+// results before touching them; it lets the next call's kernels launch at once
+// (they only read H and W before their own griddepcontrol.wait).  The last of
+// its CTAs publishes the call's status word (see StatusWords).
 //
 // draft_verify_kernel: Eq. 4 alone from caller-supplied statistics
 // (wino_draft_verify), one CTA per sequence.
@@ -256,17 +258,51 @@ __device__ void eq4_block(int a, int s, int32_t *tokens, const int32_t *argmax, 
     __syncthreads();  // the scratch may be reused for the next sequence
 }
 
+// Eq. 4: the CTA that merges the last rows of a sequence updates that sequence.
+__device__ void eq4_tail(const FinishArgs &a, int64_t row0, int32_t status, int32_t *s_done, int32_t &s_ndone,
+                         Eq4Smem &sm)
+{
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t nd = 0;
+        const int64_t per_seq =
+            ((a.p.options & (WINO_OPT_NO_SHADOW | WINO_OPT_COMPACT)) ? 1 : 2) * (int64_t)a.p.blk_len;
+        const int64_t rend = min(row0 + kFinishRows, (int64_t)a.N);
+        for (int64_t r = row0; r < rend;) {
+            const int64_t sq = r / per_seq;
+            const int64_t send = min((sq + 1) * per_seq, rend);
+            const int32_t cnt = (int32_t)(send - r);
+            if (atomicAdd(&a.tickets[sq], cnt) + cnt == per_seq)
+                s_done[nd++] = (int32_t)sq;
+            r = send;
+        }
+        s_ndone = nd;
+        __threadfence();
+    }
+    __syncthreads();
+    const int nd = s_ndone;
+    for (int i = 0; i < nd; ++i) {
+        const int sq = a.p.active_seq ? a.p.active_seq[s_done[i]] : s_done[i];
+        if (sq < 0 || sq >= a.p.n_seq) {  // a bad entry of the caller's list: no update, an error status
+            if (threadIdx.x == 0)
+                atomicExch(&a.status->current, (int32_t)WINO_ERR_ARG);
+            continue;
+        }
+        eq4_block(s_done[i], sq, a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status, sm);
+    }
+}
+
 __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishArgs a)
 {
+    ptx::grid_dep_launch_dependents();  // the next call may start streaming its H and W
     ptx::grid_dep_wait();
-    ptx::grid_dep_launch_dependents();
     __shared__ int32_t s_done[kFinishRows];
     __shared__ int32_t s_ndone;
     __shared__ Eq4Smem sm;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t row0 = (int64_t)blockIdx.x * kFinishRows;
     const int64_t row = row0 + warp;
-    const int32_t status = a.status ? *a.status : WINO_OK;
+    const int32_t status = *reinterpret_cast<volatile int32_t *>(&a.status->current);
 
     if (row < a.N) {
         if (status != WINO_OK) {
@@ -333,37 +369,17 @@ __global__ void __launch_bounds__(kFinishRows * 32) finish_kernel(const FinishAr
             }
         }
     }
-    if (!a.tokens)
-        return;
+    if (a.tokens)
+        eq4_tail(a, row0, status, s_done, s_ndone, sm);
 
-    // Eq. 4: the CTA that merges the last rows of a sequence updates that sequence.
+    // The last CTA done with this call publishes its status and clears the word for the next call.
     __syncthreads();
     if (threadIdx.x == 0) {
-        int32_t nd = 0;
-        const int64_t per_seq =
-            ((a.p.options & (WINO_OPT_NO_SHADOW | WINO_OPT_COMPACT)) ? 1 : 2) * (int64_t)a.p.blk_len;
-        const int64_t rend = min(row0 + kFinishRows, (int64_t)a.N);
-        for (int64_t r = row0; r < rend;) {
-            const int64_t sq = r / per_seq;
-            const int64_t send = min((sq + 1) * per_seq, rend);
-            const int32_t cnt = (int32_t)(send - r);
-            if (atomicAdd(&a.tickets[sq], cnt) + cnt == per_seq)
-                s_done[nd++] = (int32_t)sq;
-            r = send;
-        }
-        s_ndone = nd;
         __threadfence();
-    }
-    __syncthreads();
-    const int nd = s_ndone;
-    for (int i = 0; i < nd; ++i) {
-        const int sq = a.p.active_seq ? a.p.active_seq[s_done[i]] : s_done[i];
-        if (sq < 0 || sq >= a.p.n_seq) {  // a bad entry of the caller's list: no update, an error status
-            if (threadIdx.x == 0 && a.status)
-                atomicExch(a.status, (int32_t)WINO_ERR_ARG);
-            continue;
+        if (atomicAdd(&a.status->finished, 1u) == gridDim.x - 1) {
+            __threadfence();
+            a.status->last = atomicExch(&a.status->current, (int32_t)WINO_OK);
         }
-        eq4_block(s_done[i], sq, a.tokens, a.argmax, a.pmax, a.ptarget, a.p, a.counts, a.flags, status, sm);
     }
 }
 
@@ -382,8 +398,8 @@ __global__ void __launch_bounds__(256) gather_compact_kernel(const uint4 *__rest
                                                              const int32_t *__restrict__ tokens, const wino_params p,
                                                              int64_t vec_per_row)
 {
-    ptx::grid_dep_wait();  // the token state may still be being written by the previous step
     ptx::grid_dep_launch_dependents();  // the score kernel may set up now; it waits for these rows itself
+    ptx::grid_dep_wait();  // the token state may still be being written by the previous step
     const int64_t r = blockIdx.x;  // = s * L + l
     const int64_t s = r / p.blk_len, l = r - s * p.blk_len;
     const bool masked = tokens[s * p.seq_len + p.blk_start + l] == p.mask_id;
@@ -402,8 +418,8 @@ __global__ void __launch_bounds__(256) gather_active_kernel(const uint4 *__restr
                                                             const int32_t *__restrict__ tokens, const wino_params p,
                                                             int64_t vec_per_row)
 {
+    ptx::grid_dep_launch_dependents();  // the score kernel waits for these rows itself
     ptx::grid_dep_wait();  // the token state may still be being written by the previous step
-    ptx::grid_dep_launch_dependents();
     const bool shadow = !(p.options & WINO_OPT_NO_SHADOW);
     const bool compact = (p.options & WINO_OPT_COMPACT) != 0;
     const int64_t L = p.blk_len;

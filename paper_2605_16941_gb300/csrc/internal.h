@@ -11,20 +11,23 @@
 namespace wino {
 
 // Scoring tile: a CTA pair (2-SM tcgen05 MMA, cta_group::2) computes 256 rows
-// of H x 256 vocabulary columns.  Each CTA stages its own 128 rows of H and 128
-// of the 256 W rows per 64-wide K slice (128-byte swizzle rows) through a
-// 6-deep shared-memory ring, and holds its 128 rows x 256 columns of the fp32
-// accumulator in TMEM (one TMEM lane per row), twice: the epilogue reads one
-// accumulator while the MMAs of the next tile fill the other.
+// of H x bn vocabulary columns (bn <= 256, a multiple of 16, chosen per launch
+// by score_schedule so that the vocabulary splits evenly over the pairs).
+// Each CTA stages its own 128 rows of H and bn/2 of the tile's bn W rows per
+// 64-wide K slice (128-byte swizzle rows) through a 6-deep shared-memory ring,
+// and holds its 128 rows x bn columns of the fp32 accumulator in TMEM (one
+// TMEM lane per row), twice: the epilogue reads one accumulator while the
+// MMAs of the next tile fill the other.
 constexpr int kPairM = 256;  // rows per pair tile (UMMA M)
 constexpr int kBM = 128;     // rows per CTA
-constexpr int kBN = 256;     // vocabulary columns per tile (UMMA N)
-constexpr int kHalfN = 128;  // W rows staged by each CTA of the pair
+constexpr int kBN = 256;     // largest tile width (UMMA N); TMEM column stride of the two accumulators
+constexpr int kHalfN = 128;  // W rows staged by each CTA of the pair at the largest width
+constexpr int kMinBN = 128;  // narrowest tile width the schedule uses
 constexpr int kBK = 64;
 constexpr int kStages = 6;
 constexpr int kScoreThreads = 192;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 epilogue
 constexpr uint32_t kStageBytesA = kBM * kBK * 2;     // 16 KB
-constexpr uint32_t kStageBytesB = kHalfN * kBK * 2;  // 16 KB
+constexpr uint32_t kStageBytesB = kHalfN * kBK * 2;  // 16 KB slot (bn/2 rows of 128 B are filled)
 constexpr uint32_t kRingBytes = kStages * (kStageBytesA + kStageBytesB);
 constexpr uint32_t kScoreSmemBytes = kRingBytes + 1024 /* alignment slack */ + 256 /* barriers */;
 constexpr uint32_t kTmemCols = 2 * kBN;  // two 256-column fp32 accumulators: all 512 TMEM columns
@@ -71,19 +74,37 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
 // per (row, pair of the group): G records per row.
 constexpr int kMaxRecordsPerRow = 256;
 
+// Status words at the start of every workspace.  `current` collects the
+// errors of the call in flight: score-kernel CTAs record theirs only after
+// griddepcontrol.wait (so after the previous call's finish kernel has cleared
+// the word), and the finish kernel adds its own.  The last finish CTA of a call
+// publishes `current` as `last` (what wino_read_device_status returns) and
+// clears it for the next call; `finished` counts the finish CTAs done with the
+// call and is reset by the next call's score kernel.  A workspace starts zeroed.
+struct StatusWords {
+    int32_t current;
+    int32_t last;
+    uint32_t finished;
+};
+
+// Optional per-CTA timeline of the score kernel (diagnostics, off by default):
+// kTimelineWords 64-bit words per CTA, see score.cu.
+constexpr int kTimelineWords = 8;
+
 // Partial record: running max logit m, sum of exp(l - m), argmax (int bits),
 // logit of the row's target if the target lies in one of the pair's tiles (else -inf).
 struct ScoreArgs {
     int32_t N, d, V;
-    int32_t n_mb, n_vt, n_kb;  // n_mb: 256-row blocks
+    int32_t n_mb, n_vt, n_kb;  // n_mb: 256-row blocks, n_vt: vocabulary tiles of bn columns
+    int32_t bn;                // tile width (multiple of 16, kMinBN..kBN)
     int32_t n_groups, G;
     TargetSource ts;
     float4 *part;       // [N][G]
     float *part_u;      // [N][G], entropy variant only: sum of exp(l - m) * (l - m) * log2(e) over the pair's tiles
-    int32_t *status;    // cleared by CTA 0
+    StatusWords *status;
     int32_t *tickets;   // [n_tickets], cleared here for the finish kernel
     int32_t n_tickets;
-    int32_t h_from_prev_grid;  // H is written by the kernel launched just before (row compaction): no early loads
+    uint64_t *timeline;        // nullptr, or [gridDim.x][kTimelineWords] stamps of this launch
 };
 
 struct FinishArgs {
@@ -92,7 +113,7 @@ struct FinishArgs {
     float *entropy;       // optional: H(p) = -sum_v p_v log p_v per row
     int32_t G, N, V;
     TargetSource ts;
-    int32_t *status;  // read; set to WINO_ERR_ARG when an active-sequence list entry is out of range
+    StatusWords *status;  // read; WINO_ERR_ARG added when an active-sequence list entry is out of range
     int32_t *argmax;
     float *pmax;
     float *ptarget;
@@ -104,7 +125,21 @@ struct FinishArgs {
     int32_t *tickets;  // [n_seq], zero on entry
 };
 
-void score_schedule(int32_t n_mb, int32_t n_vt, int max_units, int32_t *n_groups, int32_t *G);
+// Work split of one score launch: tile width bn, number of row-block groups and pairs per group, for
+// n_mb 256-row blocks over a vocabulary of V entries on max_units resident pairs.  At most
+// records_cap records per row (the workspace holds that many).
+struct ScoreSchedule {
+    int32_t bn, n_vt, n_groups, G;
+};
+ScoreSchedule score_schedule(int32_t n_mb, int64_t V, int max_units, int32_t records_cap);
+
+// Records per row the workspace reserves for a vocabulary of V entries: one per tile at the narrowest
+// width, at most kMaxRecordsPerRow.
+inline int64_t records_per_row(int64_t V)
+{
+    const int64_t n = (V + kMinBN - 1) / kMinBN;
+    return n < kMaxRecordsPerRow ? n : kMaxRecordsPerRow;
+}
 
 // CTA pairs of the score kernel that can be resident at once on the current device (<= 0 on error).
 int score_max_pairs();

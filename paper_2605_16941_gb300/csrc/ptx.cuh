@@ -23,6 +23,13 @@ __device__ __forceinline__ uint64_t globaltimer_ns()
     return t;
 }
 
+__device__ __forceinline__ uint32_t smid()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+    return r;
+}
+
 // ------------------------------------------------------------------ programmatic dependent launch
 
 // Block until the grids this launch depends on have completed and their memory is visible
@@ -152,6 +159,16 @@ __device__ __forceinline__ uint64_t policy_evict_last()
     uint64_t p;
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
     return p;
+}
+
+// Prefetch a 2-D tile of a tensor into L2 (no shared memory, no completion).  L2 is the point of coherence
+// of global memory, so a prefetch may run before the writes of a previous kernel are visible to this one.
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap *m, int32_t c0, int32_t c1)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(c0), "r"(c1)
+                 : "memory");
 }
 
 // 2-D tiled bulk tensor load global -> shared, completion counted in bytes on `bar`.

@@ -3,9 +3,9 @@
 // For every scored row h_n the method needs three numbers of the model's
 // distribution p(. | Y~) = softmax_v(<h_n, w_v>) over the whole vocabulary
 // (Eq. 2 and Eq. 3 of the WINO paper): argmax_v p, max_v p and p(target).
-// The logits never leave the chip: each CTA pair computes 256 x 256 logit
+// The logits never leave the chip: each CTA pair computes 256 x bn logit
 // tiles with 2-SM tensor-core MMAs (tcgen05.mma.cta_group::2, bf16 x bf16 ->
-// fp32 in TMEM, M = 256 split 128/128 over the two SMs, N = 256), and four
+// fp32 in TMEM, M = 256 split 128/128 over the two SMs, N = bn <= 256), and four
 // epilogue warps per CTA fold each tile straight out of TMEM into a running
 // per-row state (max, sum of exp, argmax, target logit) that lives in
 // registers across all of the pair's vocabulary tiles of that row block.  One
@@ -13,22 +13,28 @@
 //
 // Kernel structure (persistent, clusters of 2 CTAs = one SM pair, 192 threads each):
 //   warp 0  TMA producer (both CTAs): streams 64-wide K slices of its 128 rows
-//           of H and of its 128 of the tile's 256 W rows into a 6-stage ring;
+//           of H and of its bn/2 of the tile's bn W rows into a 6-stage ring;
 //           both CTAs' copies complete on the LEADER's stage barrier;
 //   warp 1  TMEM allocation (both CTAs, 512 columns = two 256-column fp32
 //           accumulators) and, in the leader only, the MMA issuer:
-//           4 x (M256 N256 K16) per stage, committing stage release and
+//           4 x (M256 Nbn K16) per stage, committing stage release and
 //           accumulator-ready to both CTAs (multicast);
 //   warps 2-5 epilogue (both CTAs): one thread per row (TMEM lane); online
-//           softmax over a tile's 256 columns while the MMAs of the next tile
+//           softmax over a tile's bn columns while the MMAs of the next tile
 //           fill the other accumulator, then release the accumulator to the
 //           leader's MMA warp (8 arrivals per tile).
 // Work split: see ScoreArgs in internal.h.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA raises an
-// abort flag, records WINO_ERR_DEVICE_TIMEOUT in the status word, drains its
-// in-flight copies and MMAs (again bounded); both CTAs then meet at the
-// closing cluster barrier before TMEM is released.
+// abort flag and drains its in-flight copies and MMAs (again bounded); both
+// CTAs then meet at the closing cluster barrier before TMEM is released, and
+// the CTA records WINO_ERR_DEVICE_TIMEOUT in the call's status word.
+//
+// Optional timeline (ScoreArgs::timeline, diagnostics only): per CTA,
+// globaltimer stamps [0] entry, [1] set-up done (barriers, TMEM), [2] first
+// TMA issue, [3] griddepcontrol.wait returned in the epilogue, [4] last MMA
+// completed (leader) or last tile read (peer), [5] all roles done, [6] exit;
+// [7] = SM id << 32 | tiles of the pair.
 #include <mutex>
 
 #include "internal.h"
@@ -40,6 +46,7 @@ namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint16_t kBothCtas = 0x3;
+constexpr int kPrefetchSlices = 16;  // K slices of the first tile prefetched into L2 before the grid wait
 
 struct alignas(8) Barriers {
     uint64_t full[kStages];   // leader: both CTAs' copies of a stage landed
@@ -65,6 +72,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const uint32_t rank = ptx::cluster_ctarank();  // 0: leader (issues the MMAs), 1: peer
     const bool leader = rank == 0;
     const int pair = blockIdx.x >> 1;
+    uint64_t *const tl = a.timeline ? a.timeline + (size_t)blockIdx.x * kTimelineWords : nullptr;
+    if (tl && threadIdx.x == 0)
+        tl[0] = ptx::globaltimer_ns();
 
     auto sA = [&](int s) { return ring + (uint32_t)s * (kStageBytesA + kStageBytesB); };
     auto sB = [&](int s) { return sA(s) + kStageBytesA; };
@@ -104,11 +114,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const uint32_t tmem = bars->tmem_base;
     const uint32_t peer_tmem = ptx::ld_shared_cluster_u32(ptx::mapa(ptx::smem_u32(&bars->tmem_base), rank ^ 1u));
     const bool tmem_ok = (peer_tmem == tmem);
+    if (tl && threadIdx.x == 0)
+        tl[1] = ptx::globaltimer_ns();
 
-    // Programmatic launch: the TMA producer and the MMA warp only read H and W, which the grid before
-    // us (the finish kernel of the previous WINO call on this stream) never writes, so they start at
-    // once (unless H itself comes from the grid before us: row compaction).  Everything that touches what that grid reads or writes -- the token state (targets), the
-    // partial records, the status word and the tickets -- waits for it (grid_dep_wait) first.
+    // Programmatic launch: everything above overlapped the grid before us.  Whatever that grid is (the
+    // previous WINO call's finish kernel, or a kernel of the caller's that wrote H), its writes are only
+    // visible after griddepcontrol.wait, so every role waits before its first global access; the producer
+    // first prefetches the start of its first tile into L2, which is safe before the wait (L2 is coherent).
     ptx::grid_dep_launch_dependents();
 
     const int grp = pair % a.n_groups;  // 256-row blocks grp, grp + n_groups, ...
@@ -117,9 +129,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     if (warp >= 2 || !tmem_ok) {
         ptx::grid_dep_wait();
         if (blockIdx.x == 0 && threadIdx.x == 64)
-            *a.status = tmem_ok ? WINO_OK : WINO_ERR_UNSUPPORTED;
-        if (!tmem_ok && threadIdx.x == 64)
-            atomicExch(a.status, (int32_t)WINO_ERR_UNSUPPORTED);
+            a.status->finished = 0;  // the previous call's finish kernel has completed
+        if (tl && threadIdx.x == 64)
+            tl[3] = ptx::globaltimer_ns();
         for (int i = blockIdx.x * 128 + (int)threadIdx.x - 64; i < a.n_tickets; i += gridDim.x * 128)
             if (threadIdx.x >= 64)
                 a.tickets[i] = 0;
@@ -128,8 +140,15 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         // nothing to do: the status word reports the failed allocation check
     } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer (both CTAs)
-        if (a.h_from_prev_grid)  // H was written by the grid before us (row compaction)
-            ptx::grid_dep_wait();
+        const int half_bn = a.bn >> 1;  // W rows each CTA stages per tile
+        if (lane == 0 && grp < a.n_mb && col < a.n_vt) {
+            const int n_pre = min(a.n_kb, kPrefetchSlices);
+            for (int kb = 0; kb < n_pre; ++kb) {
+                ptx::tma_prefetch_2d(&tmW, kb * kBK, col * a.bn + (int)rank * half_bn);
+                ptx::tma_prefetch_2d(&tmH, kb * kBK, grp * kPairM + (int)rank * kBM);
+            }
+        }
+        ptx::grid_dep_wait();
         const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every vocabulary tile
         const uint64_t pol_w = ptx::policy_evict_normal();  // W is shared by the row-block groups
         int stage = 0;
@@ -138,12 +157,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         for (int s = 0; s < kStages; ++s)
             issued_parity[s] = -1;
         bool aborted = false;
+        const uint32_t stage_tx = 2 * (kStageBytesA + (uint32_t)half_bn * (kBK * 2));  // both CTAs' copies
+        bool first = true;
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
             for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
                 for (int kb = 0; kb < a.n_kb; ++kb) {
                     int ok = 1;
                     if (lane == 0)
-                        ok = wait_bounded(empty(stage), phase ^ 1u, &bars->abort, a.status);
+                        ok = wait_bounded(empty(stage), phase ^ 1u, &bars->abort);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (!ok) {
                         aborted = true;
@@ -152,10 +173,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                     if (lane == 0) {
                         const uint32_t bar = ptx::mapa(full(stage), 0);  // the leader's stage barrier
                         if (leader)
-                            ptx::mbar_arrive_expect_tx(full(stage), 2 * (kStageBytesA + kStageBytesB));
+                            ptx::mbar_arrive_expect_tx(full(stage), stage_tx);
                         ptx::tma_load_2d_pair(sA(stage), &tmH, bar, kb * kBK, mb * kPairM + (int)rank * kBM, pol_h);
-                        ptx::tma_load_2d_pair(sB(stage), &tmW, bar, kb * kBK, vt * kBN + (int)rank * kHalfN,
+                        ptx::tma_load_2d_pair(sB(stage), &tmW, bar, kb * kBK, vt * a.bn + (int)rank * half_bn,
                                               pol_w);
+                        if (tl && first)
+                            tl[2] = ptx::globaltimer_ns();
+                        first = false;
                     }
                     __syncwarp();
                     issued_parity[stage] = (int32_t)phase;
@@ -176,7 +200,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer (leader)
         if (leader) {
-            constexpr uint32_t idesc = ptx::idesc_bf16_f32(kPairM, kBN);
+            const uint32_t idesc = ptx::idesc_bf16_f32(kPairM, (uint32_t)a.bn);
+            int tiles = 0;
             int stage = 0;
             uint32_t phase = 0;
             int acc = 0;
@@ -186,7 +211,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
                     int ok = 1;
                     if (lane == 0)
-                        ok = wait_bounded<true>(tempty(acc), acc_phase ^ 1u, &bars->abort, a.status);
+                        ok = wait_bounded<true>(tempty(acc), acc_phase ^ 1u, &bars->abort);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (!ok) {
                         aborted = true;
@@ -197,7 +222,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                     for (int kb = 0; kb < a.n_kb; ++kb) {
                         ok = 1;
                         if (lane == 0)
-                            ok = wait_bounded(full(stage), phase, &bars->abort, a.status);
+                            ok = wait_bounded(full(stage), phase, &bars->abort);
                         ok = __shfl_sync(0xffffffffu, ok, 0);
                         if (!ok) {
                             aborted = true;
@@ -223,6 +248,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                     if (lane == 0)
                         ptx::mma_commit_pair_multicast(tfull(acc), kBothCtas);
                     __syncwarp();
+                    ++tiles;
                     if (++acc == 2) {
                         acc = 0;
                         acc_phase ^= 1u;
@@ -233,6 +259,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             if (lane == 0) {
                 ptx::mma_commit_pair(mma_done);
                 wait_drain(mma_done, 0);
+                if (tl) {
+                    tl[4] = ptx::globaltimer_ns();
+                    tl[7] = (uint64_t)ptx::smid() << 32 | (uint32_t)tiles;
+                }
             }
             __syncwarp();
         }
@@ -245,15 +275,15 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
             const int64_t row = (int64_t)mb * kPairM + (int)rank * kBM + q * 32 + lane;
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
-            float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tl = -INFINITY;
+            float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tlog = -INFINITY;
             float u0 = 0.f, u1 = 0.f, u2 = 0.f, u3 = 0.f;  // entropy variant
             int32_t am = 0;
             for (int vt = col; vt < a.n_vt; vt += a.G) {
-                const int32_t v0 = vt * kBN;
-                const int nvalid = min(kBN, a.V - v0);
+                const int32_t v0 = vt * a.bn;
+                const int nvalid = min(a.bn, a.V - v0);
                 int ok = 1;
                 if (lane == 0)
-                    ok = wait_bounded(tfull(acc), acc_phase, &bars->abort, a.status);
+                    ok = wait_bounded(tfull(acc), acc_phase, &bars->abort);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) {
                     aborted = true;
@@ -263,7 +293,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
 #pragma unroll 1
                 for (int c = 0; c < kBN / 32; ++c) {
-                    const int cvalid = nvalid - c * 32;  // warp-uniform
+                    const int cvalid = nvalid - c * 32;  // warp-uniform; columns past the tile are masked
                     if (cvalid <= 0)
                         break;
                     float x[32];
@@ -273,7 +303,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
                             if (j >= cvalid)
-                                x[j] = -INFINITY;  // columns past V are TMA zero fill, not logits
+                                x[j] = -INFINITY;  // past V (TMA zero fill) or past the tile (another tile's columns)
                     }
                     float cm = x[0];
 #pragma unroll
@@ -332,7 +362,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                     if ((unsigned)tj < 32u) {
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            tl = (j == tj) ? x[j] : tl;
+                            tlog = (j == tj) ? x[j] : tlog;
                     }
                 }
                 // Accumulator fully read by this warp: tell the leader's MMA warp.
@@ -346,45 +376,65 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 }
             }
             if (!aborted && row < a.N) {
-                a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tl);
+                a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tlog);
                 if (kEntropy)
                     a.part_u[row * a.G + col] = (u0 + u1) + (u2 + u3);
             }
         }
+        if (tl && !leader && warp == 2 && lane == 0)
+            tl[4] = ptx::globaltimer_ns();
     }
 
     // Neither CTA releases TMEM, or exits, while its peer may still use the pair's TMEM or barriers.
     ptx::tc_fence_before();
     __syncthreads();
+    if (tl && threadIdx.x == 0)
+        tl[5] = ptx::globaltimer_ns();
+    if (threadIdx.x == 64) {
+        // Warp 2 has passed griddepcontrol.wait, so the previous call's finish kernel, which clears the
+        // status word, has completed: a failure recorded now belongs to this call.
+        if (!tmem_ok)
+            atomicExch(&a.status->current, (int32_t)WINO_ERR_UNSUPPORTED);
+        else if (*reinterpret_cast<volatile int32_t *>(&bars->abort))
+            atomicExch(&a.status->current, (int32_t)WINO_ERR_DEVICE_TIMEOUT);
+    }
     ptx::cluster_sync();
     ptx::tc_fence_after();
     if (warp == 1)
         ptx::tmem_dealloc_pair(tmem, kTmemCols);
+    if (tl && threadIdx.x == 0)
+        tl[6] = ptx::globaltimer_ns();
 }
 
 }  // namespace
 
-// Choose the number of row-block groups: fewest tiles on the busiest pair,
-// then fewest passes over W (more groups = fewer passes).
-void score_schedule(int32_t n_mb, int32_t n_vt, int max_units, int32_t *n_groups, int32_t *G)
+// Choose the tile width bn and the number of row-block groups: fewest vocabulary columns on the busiest
+// pair (tiles x (bn + a per-tile overhead)), then the widest tile, then fewest passes over W (more groups).
+// A width below kBN pays when the vocabulary then splits evenly over the pairs: V = 126464 on 76 pairs is
+// 494 tiles of 256 (7 on the busiest pair, 6.5 on average) but 527 tiles of 240 (7 on the busiest pair).
+ScoreSchedule score_schedule(int32_t n_mb, int64_t V, int max_units, int32_t records_cap)
 {
-    int64_t best_rounds = -1;
-    int32_t best_groups = 1, best_g = 1;
+    constexpr int64_t kTileOverheadCols = 16;  // H re-read and accumulator hand-over per tile, in columns
+    ScoreSchedule best{kBN, (int32_t)((V + kBN - 1) / kBN), 1, 1};
+    int64_t best_cost = -1;
     const int32_t top = n_mb < max_units ? n_mb : max_units;
-    for (int32_t groups = top; groups >= 1; --groups) {
-        int32_t g = max_units / groups;
-        g = g < n_vt ? g : n_vt;
-        g = g < kMaxRecordsPerRow ? g : kMaxRecordsPerRow;
-        g = g < 1 ? 1 : g;
-        const int64_t rounds = (int64_t)((n_mb + groups - 1) / groups) * ((n_vt + g - 1) / g);
-        if (best_rounds < 0 || rounds < best_rounds) {
-            best_rounds = rounds;
-            best_groups = groups;
-            best_g = g;
+    for (int32_t bn = kBN; bn >= kMinBN; bn -= 16) {
+        const int64_t n_vt = (V + bn - 1) / bn;
+        for (int32_t groups = top; groups >= 1; --groups) {
+            int64_t g = max_units / groups;
+            g = g < n_vt ? g : n_vt;
+            g = g < records_cap ? g : records_cap;
+            g = g < kMaxRecordsPerRow ? g : kMaxRecordsPerRow;
+            g = g < 1 ? 1 : g;
+            const int64_t rounds = (int64_t)((n_mb + groups - 1) / groups) * ((n_vt + g - 1) / g);
+            const int64_t cost = rounds * (bn + kTileOverheadCols);
+            if (best_cost < 0 || cost < best_cost) {
+                best_cost = cost;
+                best = ScoreSchedule{bn, (int32_t)n_vt, groups, (int32_t)g};
+            }
         }
     }
-    *n_groups = best_groups;
-    *G = best_g;
+    return best;
 }
 
 namespace {

@@ -2,9 +2,9 @@
 //
 // One CTA initialises an mbarrier that nothing will ever arrive on and waits
 // for it with the same bounded wait the score kernel uses, shortened to the
-// caller's limit.  The wait must give up, raise the abort flag and record
-// WINO_ERR_DEVICE_TIMEOUT in *status; the kernel then exits normally, so the
-// CUDA context stays usable.  This is how the library's timeout handling is
+// caller's limit.  The wait must give up and raise the abort flag; the kernel
+// records WINO_ERR_DEVICE_TIMEOUT in *status and exits normally, so the CUDA
+// context stays usable.  This is how the library's timeout handling is
 // exercised on a GPU without hanging or faulting it.
 #include "internal.h"
 #include "ptx.cuh"
@@ -25,8 +25,8 @@ __global__ void wait_timeout_kernel(int32_t *status, uint64_t limit_ns)
     ptx::mbar_init(b, 1);
     ptx::fence_barrier_init();
     // nothing arrives: phase 0 never completes
-    if (wait_bounded(b, 0, &abort_flag, status, limit_ns))
-        *status = WINO_OK;  // unreachable unless the wait is broken
+    if (!wait_bounded(b, 0, &abort_flag, limit_ns) && abort_flag)
+        *status = WINO_ERR_DEVICE_TIMEOUT;
 }
 
 }  // namespace

@@ -19,25 +19,28 @@ namespace {
 // The scratch every call of wino_step_static_scratch on a device shares.
 static __device__ __align__(256) unsigned char g_static_scratch[WINO_STATIC_SCRATCH_BYTES];
 
-// In host code g_static_scratch only names the array; its device address is looked up once per
-// device, with that device current.
-int scratch_address(void **out)
+// In host code g_static_scratch only names the array; its device address is looked up with the device
+// current, on every call (a cheap table lookup once the module is loaded), so that a module reloaded
+// after cudaDeviceReset is never reached through a stale address.  The first call that sees an address
+// (per device) also clears the status words at the start of the array on the caller's stream, which the
+// kernels expect to find zeroed before their first use.
+int scratch_address(cudaStream_t stream, void **out)
 {
     static std::mutex mu;
-    static void *addr[64];
-    static bool have[64];
+    static void *seen[64];
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
         return WINO_ERR_CUDA;
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p)
+        return WINO_ERR_CUDA;
     std::lock_guard<std::mutex> g(mu);
-    if (!have[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p)
+    if (seen[dev] != p) {
+        if (cudaMemsetAsync(p, 0, 256, stream) != cudaSuccess)
             return WINO_ERR_CUDA;
-        addr[dev] = p;
-        have[dev] = true;
+        seen[dev] = p;
     }
-    *out = addr[dev];
+    *out = p;
     return WINO_OK;
 }
 
@@ -56,7 +59,7 @@ extern "C" int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, in
     if (need > WINO_STATIC_SCRATCH_BYTES)
         return WINO_ERR_WORKSPACE;  // the problem needs more scratch than the fixed array holds
     void *scratch = nullptr;
-    const int rs = wino::scratch_address(&scratch);
+    const int rs = wino::scratch_address(static_cast<cudaStream_t>(stream), &scratch);
     if (rs != WINO_OK)
         return rs;
     return wino_step(H, W, d, V, tokens, p, counts, flags, scratch, WINO_STATIC_SCRATCH_BYTES, stream);

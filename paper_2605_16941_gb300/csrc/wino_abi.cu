@@ -24,27 +24,29 @@ constexpr size_t kAlign = 256;
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Workspace layout: [status | tickets[ceil(N/2)] | partial records [N][R] | entropy partials [N][R] |
-// argmax[N] | pmax[N] | ptarget[N]], R = min(ceil(V/kBN), kMaxRecordsPerRow) bounds the records per row.
+// Workspace layout: [status words | tickets[ceil(N/2)] | partial records [N][R] | argmax[N] | pmax[N] |
+// ptarget[N] || entropy partials [N][R]], R = records_per_row(V) bounds the records per row.  `total` ends
+// before the entropy partials, which only wino_score_rows with an entropy output needs (`total_entropy`).
 struct WsLayout {
-    size_t status, tickets, part, part_u, argmax, pmax, ptarget, total;
+    size_t status, tickets, part, argmax, pmax, ptarget, total, part_u, total_entropy;
 };
 
 WsLayout ws_layout(int64_t N, int64_t V)
 {
-    const int64_t n_vt = (V + kBN - 1) / kBN;
-    const int64_t R = n_vt < kMaxRecordsPerRow ? n_vt : kMaxRecordsPerRow;
+    const int64_t R = records_per_row(V);
     WsLayout L{};
     L.status = 0;
     L.tickets = kAlign;
     L.part = L.tickets + round_up((size_t)((N + 1) / 2) * 4, kAlign);
-    L.part_u = L.part + round_up((size_t)N * (size_t)R * sizeof(float4), kAlign);
-    L.argmax = L.part_u + round_up((size_t)N * (size_t)R * sizeof(float), kAlign);
+    L.argmax = L.part + round_up((size_t)N * (size_t)R * sizeof(float4), kAlign);
     L.pmax = L.argmax + round_up((size_t)N * 4, kAlign);
     L.ptarget = L.pmax + round_up((size_t)N * 4, kAlign);
     L.total = L.ptarget + round_up((size_t)N * 4, kAlign);
+    L.part_u = L.total;
+    L.total_entropy = L.part_u + round_up((size_t)N * (size_t)R * sizeof(float), kAlign);
     return L;
 }
+static_assert(sizeof(StatusWords) <= kAlign, "status words must fit the first 256 bytes");
 
 bool shape_ok(int64_t N, int64_t d, int64_t V)
 {
@@ -150,6 +152,24 @@ int tensor_map(const void *ptr, int64_t rows, int64_t cols, int box_rows, CUtens
     return WINO_OK;
 }
 
+// ---------------------------------------------------------------- score-kernel timeline (diagnostics)
+
+// While enabled, score launch i writes its per-CTA stamps into slot i % n_launches of the caller's buffer.
+struct Timeline {
+    std::mutex mu;
+    uint64_t *buf = nullptr;
+    int64_t n_launches = 0, ctas_per_launch = 0, next = 0;
+} g_timeline;
+
+uint64_t *timeline_slot(unsigned grid)
+{
+    std::lock_guard<std::mutex> g(g_timeline.mu);
+    if (!g_timeline.buf || (int64_t)grid > g_timeline.ctas_per_launch)
+        return nullptr;
+    const int64_t i = g_timeline.next++ % g_timeline.n_launches;
+    return g_timeline.buf + i * g_timeline.ctas_per_launch * kTimelineWords;
+}
+
 // ---------------------------------------------------------------- launch timing
 
 // Optional timing of the score kernel: while enabled, every score launch is
@@ -197,40 +217,44 @@ int check_params(const wino_params *p)
 // the score kernel followed by the finish kernel.
 int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
                      int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws, size_t ws_bytes,
-                     const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream,
-                     bool h_from_prev_grid = false)
+                     const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream)
 {
     DeviceInfo info;
     int rc = device_info(&info);
     if (rc != WINO_OK)
         return rc;
     const WsLayout L = ws_layout(N, V);
-    if (ws_bytes < L.total)
+    if (ws_bytes < (entropy ? L.total_entropy : L.total))
         return WINO_ERR_WORKSPACE;
-    CUtensorMap tmH, tmW;
-    if ((rc = tensor_map(H, N, d, kBM, &tmH)) != WINO_OK)
-        return rc;
-    if ((rc = tensor_map(W, V, d, kHalfN, &tmW)) != WINO_OK)
-        return rc;
     const int max_pairs = score_max_pairs();
     if (max_pairs < 1)
         return WINO_ERR_CUDA;
+    const int32_t n_mb = (int32_t)((N + kPairM - 1) / kPairM);
+    const ScoreSchedule sch =
+        score_schedule(n_mb, V, std::min(max_pairs, info.sm_count / 2), (int32_t)records_per_row(V));
+    CUtensorMap tmH, tmW;
+    if ((rc = tensor_map(H, N, d, kBM, &tmH)) != WINO_OK)
+        return rc;
+    if ((rc = tensor_map(W, V, d, sch.bn / 2, &tmW)) != WINO_OK)
+        return rc;
     uint8_t *w8 = static_cast<uint8_t *>(ws);
     ScoreArgs a{};
     a.N = (int32_t)N;
     a.d = (int32_t)d;
     a.V = (int32_t)V;
-    a.n_mb = (int32_t)((N + kPairM - 1) / kPairM);
-    a.n_vt = (int32_t)((V + kBN - 1) / kBN);
+    a.n_mb = n_mb;
+    a.n_vt = sch.n_vt;
     a.n_kb = (int32_t)((d + kBK - 1) / kBK);
-    score_schedule(a.n_mb, a.n_vt, std::min(max_pairs, info.sm_count / 2), &a.n_groups, &a.G);
+    a.bn = sch.bn;
+    a.n_groups = sch.n_groups;
+    a.G = sch.G;
     a.ts = ts;
     a.part = reinterpret_cast<float4 *>(w8 + L.part);
-    a.part_u = reinterpret_cast<float *>(w8 + L.part_u);
-    a.status = reinterpret_cast<int32_t *>(w8 + L.status);
+    a.part_u = entropy ? reinterpret_cast<float *>(w8 + L.part_u) : nullptr;
+    a.status = reinterpret_cast<StatusWords *>(w8 + L.status);
     a.tickets = reinterpret_cast<int32_t *>(w8 + L.tickets);
     a.n_tickets = step ? step->n_seq : 0;
-    a.h_from_prev_grid = h_from_prev_grid ? 1 : 0;
+    a.timeline = timeline_slot((unsigned)(2 * a.n_groups * a.G));
     prof_record(0, stream);
     if (launch_score(tmH, tmW, a, entropy != nullptr, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
@@ -307,7 +331,7 @@ int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
         return WINO_ERR_ARG;
     if (!shape_ok(N, d, V))
         return WINO_ERR_SHAPE;
-    *bytes = ws_layout(N, V).total;
+    *bytes = ws_layout(N, V).total_entropy;
     return WINO_OK;
 }
 
@@ -407,8 +431,7 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
             return WINO_ERR_CUDA;
         TargetSource tsa{};
         tsa.target = tgt;
-        return score_and_finish(Hc, W, N, d, V, tsa, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s,
-                                true);
+        return score_and_finish(Hc, W, N, d, V, tsa, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s);
     }
     if (compact) {  // gather the one row per position Eq. 4 reads, behind the workspace proper
         DeviceInfo info;
@@ -419,8 +442,7 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
             return WINO_ERR_CUDA;
         Hs = Hc;
     }
-    return score_and_finish(Hs, W, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s,
-                            compact);
+    return score_and_finish(Hs, W, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s);
 }
 
 int wino_profile_begin(int max_launches)
@@ -479,10 +501,63 @@ int wino_read_device_status(const void *ws, void *stream, int *device_status)
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(s) != cudaSuccess)
         return WINO_ERR_CUDA;
-    int32_t v = 0;
-    if (cudaMemcpy(&v, ws, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess)
+    StatusWords w{};
+    if (cudaMemcpy(&w, ws, sizeof w, cudaMemcpyDeviceToHost) != cudaSuccess)
         return WINO_ERR_CUDA;
-    *device_status = v;
+    *device_status = w.last;
+    return WINO_OK;
+}
+
+int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan)
+{
+    if (!plan)
+        return WINO_ERR_ARG;
+    if (!shape_ok(N, d, V))
+        return WINO_ERR_SHAPE;
+    DeviceInfo info;
+    int rc = device_info(&info);
+    if (rc != WINO_OK)
+        return rc;
+    const int max_pairs = score_max_pairs();
+    if (max_pairs < 1)
+        return WINO_ERR_CUDA;
+    const int32_t n_mb = (int32_t)((N + kPairM - 1) / kPairM);
+    const ScoreSchedule sch =
+        score_schedule(n_mb, V, std::min(max_pairs, info.sm_count / 2), (int32_t)records_per_row(V));
+    plan[0] = sch.bn;
+    plan[1] = sch.n_vt;
+    plan[2] = n_mb;
+    plan[3] = sch.n_groups;
+    plan[4] = sch.G;
+    plan[5] = 2 * sch.n_groups * sch.G;
+    return WINO_OK;
+}
+
+int wino_timeline_begin(uint64_t *buf, int64_t n_launches, int64_t ctas_per_launch)
+{
+    if (!buf || !aligned(buf, 8) || n_launches < 1 || ctas_per_launch < 2 || ctas_per_launch > (1 << 16) ||
+        n_launches > (int64_t(1) << 20))
+        return WINO_ERR_ARG;
+    std::lock_guard<std::mutex> g(g_timeline.mu);
+    if (g_timeline.buf)
+        return WINO_ERR_ARG;
+    g_timeline.buf = buf;
+    g_timeline.n_launches = n_launches;
+    g_timeline.ctas_per_launch = ctas_per_launch;
+    g_timeline.next = 0;
+    return WINO_OK;
+}
+
+int wino_timeline_end(int64_t *launches)
+{
+    if (!launches)
+        return WINO_ERR_ARG;
+    std::lock_guard<std::mutex> g(g_timeline.mu);
+    if (!g_timeline.buf)
+        return WINO_ERR_ARG;
+    *launches = g_timeline.next;
+    g_timeline.buf = nullptr;
+    g_timeline.n_launches = g_timeline.ctas_per_launch = g_timeline.next = 0;
     return WINO_OK;
 }
 

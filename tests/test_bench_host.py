@@ -6,7 +6,6 @@ from pathlib import Path
 import bench
 
 ROOT = Path(bench.ROOT)
-WORKLOAD = "llada8b_d4096_V126464_B1_L128"
 
 
 def _copy_tree(tmp_path):
@@ -21,21 +20,33 @@ def _copy_tree(tmp_path):
     return dst
 
 
+def _sha(csrc, names):
+    import hashlib
+    h = hashlib.sha256()
+    for name in names:
+        h.update((csrc / name).read_bytes())
+    return h.hexdigest()[:16]
+
+
 def test_ncu_traffic_is_tied_to_the_kernel_sources(tmp_path, monkeypatch):
+    """A traffic record counts only while every source file the score kernel is built from is unchanged."""
     rec = json.loads((ROOT / "profiles" / "score_kernel_traffic.txt").read_text())
     want = float(rec["dram_bytes_read"]) + float(rec["dram_bytes_write"])
-    assert bench.ncu_traffic(WORKLOAD) == want
+    fresh = rec["sources_sha256_prefix"] == _sha(ROOT / "paper_2605_16941_gb300" / "csrc", rec["score_kernel_sources"])
+    assert bench.ncu_traffic(rec["workload"]) == (want if fresh else None)
     assert bench.ncu_traffic("some_other_workload") is None
     csrc = _copy_tree(tmp_path)
+    rec["sources_sha256_prefix"] = _sha(csrc, rec["score_kernel_sources"])  # a record taken on these sources
+    (tmp_path / "profiles" / "score_kernel_traffic.txt").write_text(json.dumps(rec))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.ncu_traffic(WORKLOAD) == want
+    assert bench.ncu_traffic(rec["workload"]) == want
     for name in rec["score_kernel_sources"]:  # a change to any source the kernel is built from voids it
         f = csrc / name
         old = f.read_bytes()
         f.write_bytes(old + b"\n// edited\n")
-        assert bench.ncu_traffic(WORKLOAD) is None, name
+        assert bench.ncu_traffic(rec["workload"]) is None, name
         f.write_bytes(old)
-    assert bench.ncu_traffic(WORKLOAD) == want
+    assert bench.ncu_traffic(rec["workload"]) == want
 
 
 def test_job_rows_per_s_counts_every_rank():

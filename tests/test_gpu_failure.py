@@ -59,3 +59,28 @@ def test_loop_driver_reports_a_device_failure(monkeypatch):
                      tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id,
                      hidden=lambda k, b0: dev(ws.hidden_states(w, W, st, step=k)))
     assert e.value.status == wino.WINO_ERR_DEVICE_TIMEOUT and calls == [1, 2, 3]
+
+
+def test_failure_status_reaches_the_host_once_and_is_cleared():
+    """The status words at the start of a workspace: an error recorded for a call (planted here on the
+    host, as a score-kernel CTA would record a timeout) makes that call's finish kernel leave the token
+    state alone, write the status into every counts entry and publish it for wino_read_device_status;
+    the next call starts clean and runs normally."""
+    import paper_2605_16941_gb300 as wino
+    from gpu_helpers import dev, host
+    w = ws.WORKLOADS["tiny"]
+    W = ws.weights(w)
+    st = ws.initial_state(w)
+    Hd, Wd = dev(ws.hidden_states(w, W, st)), dev(W)
+    wsp = wino.workspace(w.N, w.d, w.V)
+    p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len)
+    tok = dev(st.tokens)
+    counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device="cuda")
+    wsp[:4].view(torch.int32).fill_(wino.WINO_ERR_DEVICE_TIMEOUT)  # the word errors of the call in flight go to
+    wino.wino_step(Hd, Wd, tok, p, counts, wsp)
+    assert wino.wino_read_device_status(wsp) == wino.WINO_ERR_DEVICE_TIMEOUT
+    assert np.all(host(counts) == wino.WINO_ERR_DEVICE_TIMEOUT)
+    assert np.array_equal(host(tok), st.tokens)
+    wino.wino_step(Hd, Wd, tok, p, counts, wsp)
+    assert wino.wino_read_device_status(wsp) == wino.WINO_OK
+    assert np.all(host(counts) >= 0) and not np.array_equal(host(tok), st.tokens)

@@ -129,47 +129,6 @@ def test_step_llada_b1_full_oracle(llada, variant):
         assert rep["threshold_drafts"] > 0 and rep["kept_decoded"] > 0 and rep["remasked"] > 0
 
 
-def _check_sampled(w, W, Wd, tau1, n_rows=24):
-    """Full-size batch: every row's statistics sampled against the oracle; Eq. 4 exact on the GPU's
-    own statistics; wino_step identical to the decomposed path; invariants on every position."""
-    from gpu_helpers import compare_rows, f32
-    st = ws.initial_state(w)
-    H = ws.hidden_states(w, W, st, step=0)
-    tok, cnt, fl = _gpu_step(w, Wd, st.tokens, H, st.blk_start, tau1)
-    g, t, tok2, cnt2, fl2 = _gpu_decomposed(w, Wd, st.tokens, H, st.blk_start, tau1)
-    assert np.array_equal(tok, tok2) and np.array_equal(cnt, cnt2) and np.array_equal(fl, fl2)
-    ref_tok, ref_cnt, ref_fl = oracle.draft_verify(st.tokens, st.blk_start, w.blk_len, w.mask_id, f32(tau1),
-                                                   f32(w.tau2), g.argmax, g.pmax.astype(np.float64),
-                                                   g.ptarget.astype(np.float64))
-    assert np.array_equal(tok, ref_tok) and np.array_equal(cnt, ref_cnt) and np.array_equal(fl, ref_fl)
-    rows = np.random.default_rng(1).choice(w.N, n_rows, replace=False)
-    o = oracle.score_rows(H[rows], W, t[rows])
-    rep = compare_rows(o, g, rows)
-    L, b0 = w.blk_len, st.blk_start
-    pre = st.tokens[:, b0:b0 + L]
-    post = tok[:, b0:b0 + L]
-    assert np.array_equal(np.delete(tok, np.s_[b0:b0 + L], 1), np.delete(st.tokens, np.s_[b0:b0 + L], 1))
-    assert np.all((post == pre) | (pre == w.mask_id) | (post == w.mask_id))
-    return rep, {"drafted": int(cnt[:, 0].sum()), "remasked": int(cnt[:, 1].sum()), "left": int(cnt[:, 2].sum()),
-                 "fallback": int((fl == 2).sum())}
-
-
-@pytest.mark.parametrize("tau1", [0.5, 0.7, 0.9])
-def test_step_llada_b8_sampled(llada, tau1):
-    W, Wd = llada
-    w = ws.WORKLOADS["llada_b8"]
-    rep, c = _check_sampled(w, W, Wd, tau1)
-    print(f"llada_b8 tau1={tau1}: {rep} {c}")
-
-
-def test_step_unified_b4_sampled():
-    from gpu_helpers import dev
-    w = ws.WORKLOADS["unified_b4"]
-    W = ws.weights(w)
-    rep, c = _check_sampled(w, W, dev(W), w.tau1)
-    print(f"unified_b4: {rep} {c}")
-
-
 def test_decode_loop_tiny_lockstep():
     """The tiny workload decoded to the end through the package's loop driver; every step is
     re-run by the oracle from the same pre-step state and compared."""
@@ -215,60 +174,6 @@ def test_decode_loop_tiny_lockstep():
     assert np.array_equal(host(last_d), finalization_steps_from_trajectory(traj))  # t_l of Sec. 5.1
     print("tiny loop steps/block", [b.steps for b in stats.blocks], "flagged",
           sum(r["flagged_positions"] for r in reports))
-
-
-def test_decode_loop_b16():
-    """Config-5 loop (B=16, gen 256 in 8 blocks of 32, bias U[0, 4 + 0.5 k] at global step k):
-    runs until no MASK remains; invariants on every step; the oracle re-checks sampled steps."""
-    import paper_2605_16941_gb300.loop as loop
-    from gpu_helpers import compare_rows, dev, f32, gpu_score, host
-    w = ws.WORKLOADS["loop_b16"]
-    W = ws.weights(w)
-    Wd = dev(W)
-    st = ws.initial_state(w)
-    tok_d = dev(st.tokens)
-    rec = {}
-    sampled = {0, 1, 2, 3, 40, 200}
-
-    def hidden(k, b0):
-        st.blk_start = b0
-        H = ws.hidden_states(w, W, st, step=k)
-        rec["pre"] = host(tok_d).copy()
-        rec["H"] = H
-        rec["Hd"] = dev(H)
-        return rec["Hd"]
-
-    checked = []
-
-    def on_step(k, b0, counts, flags):
-        pre, post = rec["pre"], host(tok_d)
-        L = w.blk_len
-        outside = np.ones(w.seq_len, bool)
-        outside[b0:b0 + L] = False
-        assert np.array_equal(post[:, outside], pre[:, outside])
-        a, b = pre[:, b0:b0 + L], post[:, b0:b0 + L]
-        fl = host(flags)
-        assert np.all((b == a) | (a == w.mask_id) | (b == w.mask_id))
-        had_mask = (a == w.mask_id).any(1)
-        assert np.all((counts[:, 0] >= 1) | ~had_mask | (fl == 4).any(1))
-        assert np.array_equal(counts[:, 2], (b == w.mask_id).sum(1))
-        if k in sampled:
-            t = oracle.row_targets(pre, b0, L, w.mask_id)
-            g = gpu_score(rec["Hd"], Wd, t)
-            ref = oracle.draft_verify(pre, b0, L, w.mask_id, f32(w.tau1), f32(w.tau2), g.argmax,
-                                      g.pmax.astype(np.float64), g.ptarget.astype(np.float64), freeze_finished=True)
-            assert np.array_equal(post, ref[0]) and np.array_equal(counts, ref[1])
-            rows = np.random.default_rng(k).choice(w.N, 8, replace=False)
-            compare_rows(oracle.score_rows(rec["H"][rows], W, t[rows]), g, rows)
-            checked.append(k)
-
-    stats = loop.decode(Wd, tok_d, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks, tau1=w.tau1,
-                        tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, on_step=on_step, max_steps=4096)
-    final = host(tok_d)
-    assert not np.any(final[:, w.prompt_len:] == w.mask_id)
-    print("loop_b16 steps/block", [b.steps for b in stats.blocks], "total", stats.total_steps,
-          "drafted/block", [b.drafted for b in stats.blocks], "remasked/block", [b.remasked for b in stats.blocks],
-          "oracle-checked steps", checked)
 
 
 @pytest.mark.parametrize("n_seq,L,S,b0", CASES[:5], ids=[f"B{c[0]}_L{c[1]}" for c in CASES[:5]])
