@@ -92,6 +92,12 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
 
+    def wait_first(self, timeout_s: float = 10.0):
+        """Return once nvidia-smi has printed a sample (its start-up is then over), or after the timeout."""
+        t0 = time.time()
+        while self.proc and not self.samples and time.time() - t0 < timeout_s and self.proc.poll() is None:
+            time.sleep(0.05)
+
     def stop(self):
         if self.proc:
             self.proc.terminate()
@@ -472,7 +478,9 @@ def run_wino(args, rank, world, local_rank):
         torch.cuda.synchronize(dev)
 
     clocks = ClockSampler(gpu_uuid(dev)) if rank == 0 else None
-    time.sleep(0.3 if clocks else 0)
+    if clocks:
+        clocks.wait_first()  # nvidia-smi's start-up must not overlap the timed region
+        time.sleep(0.2)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()

@@ -331,11 +331,13 @@ WINO_API int wino_timeline_end(int64_t *launches);
 
 /*
  * How a score launch of N rows over V entries is split on the current device
- * (diagnostics; the paper has no counterpart): plan (host int32[6]) receives
+ * (diagnostics; the paper has no counterpart): plan (host int32[8]) receives
  * the tile width bn, the vocabulary tiles n_vt = ceil(V / bn), the 256-row
  * blocks n_mb, the row-block groups, the CTA pairs per group G (= records per
- * row) and the grid size in CTAs.  Pair c of the launch serves row blocks
- * c % groups (+ groups, ...) and, within each, tiles c / groups (+ G, ...).
+ * row), the grid size in CTAs, 1 if tiles are taken two per pass (one staging
+ * of H for both) else 0, and the shared-memory ring stages.  Pair c of the
+ * launch serves row blocks c % groups (+ groups, ...) and, within each, tiles
+ * c / groups (+ G, ...).
  */
 WINO_API int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan);
 

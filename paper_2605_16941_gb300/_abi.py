@@ -276,9 +276,9 @@ def wino_profile_end() -> tuple[float, int]:
 
 def wino_score_plan(N: int, d: int, V: int) -> dict:
     """The score kernel's work split for N rows over V entries on the current device."""
-    out = (C.c_int32 * 6)()
+    out = (C.c_int32 * 8)()
     _check(lib().wino_score_plan(int(N), int(d), int(V), out), "wino_score_plan")
-    return dict(zip(("bn", "n_vt", "n_mb", "n_groups", "G", "ctas"), list(out)))
+    return dict(zip(("bn", "n_vt", "n_mb", "n_groups", "G", "ctas", "two", "stages"), list(out)))
 
 
 def wino_timeline_begin(buf, n_launches: int, ctas_per_launch: int) -> None:

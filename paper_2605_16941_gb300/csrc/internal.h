@@ -12,25 +12,33 @@ namespace wino {
 
 // Scoring tile: a CTA pair (2-SM tcgen05 MMA, cta_group::2) computes 256 rows
 // of H x bn vocabulary columns (bn <= 256, a multiple of 16, chosen per launch
-// by score_schedule so that the vocabulary splits evenly over the pairs).
-// Each CTA stages its own 128 rows of H and bn/2 of the tile's bn W rows per
-// 64-wide K slice (128-byte swizzle rows) through a 6-deep shared-memory ring,
-// and holds its 128 rows x bn columns of the fp32 accumulator in TMEM (one
-// TMEM lane per row), twice: the epilogue reads one accumulator while the
-// MMAs of the next tile fill the other.
+// by score_schedule so that the vocabulary splits evenly over the pairs).  Per
+// 64-wide K slice each CTA stages its own 128 rows of H and bn/2 of the tile's
+// bn W rows (128-byte swizzle rows) in a ring of shared-memory stages, and
+// holds its 128 rows x bn columns of the fp32 accumulator in TMEM (one TMEM
+// lane per row).  Two fp32 accumulators fill TMEM's 512 columns; a launch uses
+// them in one of two modes (ScoreArgs::two):
+//   single tiles: the accumulators alternate, so the epilogue of one tile
+//     overlaps the MMAs of the next; stages of 16 KB + bn*64 B, up to 7 of them
+//     (the most bytes in flight, for shapes bound by the W stream from HBM);
+//   two-tile passes: a stage holds one H slice and the slices of two tiles,
+//     multiplied into both accumulators, so H is staged once per two tiles
+//     (a quarter fewer bytes delivered per SM and MMA, for tensor-bound shapes).
 constexpr int kPairM = 256;  // rows per pair tile (UMMA M)
 constexpr int kBM = 128;     // rows per CTA
 constexpr int kBN = 256;     // largest tile width (UMMA N); TMEM column stride of the two accumulators
-constexpr int kHalfN = 128;  // W rows staged by each CTA of the pair at the largest width
 constexpr int kMinBN = 128;  // narrowest tile width the schedule uses
 constexpr int kBK = 64;
-constexpr int kStages = 6;
+constexpr int kMaxStages = 7;
 constexpr int kScoreThreads = 192;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 epilogue
-constexpr uint32_t kStageBytesA = kBM * kBK * 2;     // 16 KB
-constexpr uint32_t kStageBytesB = kHalfN * kBK * 2;  // 16 KB slot (bn/2 rows of 128 B are filled)
-constexpr uint32_t kRingBytes = kStages * (kStageBytesA + kStageBytesB);
-constexpr uint32_t kScoreSmemBytes = kRingBytes + 1024 /* alignment slack */ + 256 /* barriers */;
+constexpr uint32_t kStageBytesA = kBM * kBK * 2;  // 16 KB of H per stage
+constexpr uint32_t kScoreSmemMax = 227u * 1024u;  // the most dynamic shared memory a CTA may have
+constexpr uint32_t kSmemOverhead = 1024 /* ring alignment slack */ + 256 /* barriers */;
+constexpr uint32_t kRingCapacity = kScoreSmemMax - kSmemOverhead;
 constexpr uint32_t kTmemCols = 2 * kBN;  // two 256-column fp32 accumulators: all 512 TMEM columns
+
+// W bytes one CTA stages per K slice of a tile of width bn (bn/2 rows of 128 B; a multiple of 1 KB).
+__host__ __device__ constexpr uint32_t stage_bytes_w(int bn) { return (uint32_t)(bn / 2) * kBK * 2; }
 
 constexpr int kMaxBlkLen = 1024;
 
@@ -67,7 +75,7 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
 
 // Work split of the score kernel.  The 256-row blocks are spread over n_groups
 // groups of G CTA pairs; pair c serves row blocks c % n_groups (+ n_groups, ...)
-// and, within each, vocabulary tiles c / n_groups (+ G, ...).  The G pairs of a
+// and, within each, vocabulary tiles c / n_groups (+ G, ...), two per pass.  The G pairs of a
 // group walk the vocabulary side by side, so all groups read the same W tiles
 // at the same time (W streams from HBM about once), and each CTA keeps its
 // running softmax state per row across its tiles and writes ONE partial record
@@ -97,6 +105,9 @@ struct ScoreArgs {
     int32_t N, d, V;
     int32_t n_mb, n_vt, n_kb;  // n_mb: 256-row blocks, n_vt: vocabulary tiles of bn columns
     int32_t bn;                // tile width (multiple of 16, kMinBN..kBN)
+    int32_t two;               // 1: two-tile passes, 0: single tiles (see above)
+    int32_t stages;            // ring stages, 2..kMaxStages
+    uint32_t stage_bytes;      // 16 KB + (1 + two) * stage_bytes_w(bn)
     int32_t n_groups, G;
     TargetSource ts;
     float4 *part;       // [N][G]
@@ -130,6 +141,8 @@ struct FinishArgs {
 // records_cap records per row (the workspace holds that many).
 struct ScoreSchedule {
     int32_t bn, n_vt, n_groups, G;
+    int32_t two, stages;
+    uint32_t stage_bytes;
 };
 ScoreSchedule score_schedule(int32_t n_mb, int64_t V, int max_units, int32_t records_cap);
 

@@ -3,26 +3,39 @@
 // For every scored row h_n the method needs three numbers of the model's
 // distribution p(. | Y~) = softmax_v(<h_n, w_v>) over the whole vocabulary
 // (Eq. 2 and Eq. 3 of the WINO paper): argmax_v p, max_v p and p(target).
-// The logits never leave the chip: each CTA pair computes 256 x bn logit
-// tiles with 2-SM tensor-core MMAs (tcgen05.mma.cta_group::2, bf16 x bf16 ->
-// fp32 in TMEM, M = 256 split 128/128 over the two SMs, N = bn <= 256), and four
-// epilogue warps per CTA fold each tile straight out of TMEM into a running
-// per-row state (max, sum of exp, argmax, target logit) that lives in
-// registers across all of the pair's vocabulary tiles of that row block.  One
-// partial record per (row, pair) goes to the workspace; finish.cu merges them.
+// The logits never leave the chip: each CTA pair computes logit tiles of 256
+// rows x bn vocabulary columns with 2-SM tensor-core MMAs
+// (tcgen05.mma.cta_group::2, bf16 x bf16 -> fp32 in TMEM, M = 256 split
+// 128/128 over the two SMs, N = bn <= 256), and four epilogue warps per CTA
+// fold each tile straight out of TMEM into a running per-row state (max, sum
+// of exp, argmax, target logit) that lives in registers across all of the
+// pair's vocabulary tiles of that row block.  One partial record per
+// (row, pair) goes to the workspace; finish.cu merges them.
+//
+// Two modes (ScoreArgs::two, chosen per launch by score_schedule):
+//   single tiles, for shapes bound by the W stream from HBM (one 256-row
+//     block): the two accumulators alternate between consecutive tiles, so
+//     the epilogue of one tile overlaps the MMAs of the next, and the ring has
+//     up to 7 stages, the most W bytes in flight per SM;
+//   two-tile passes, for tensor-bound shapes: every K slice of H is staged
+//     once and multiplied with the slices of two tiles into both accumulators,
+//     a quarter fewer bytes delivered per SM and MMA.  The accumulators then
+//     fill TMEM, so a pass's MMAs into the first accumulator start as soon as
+//     the epilogue has read it, and its MMAs into the second accumulator for
+//     the first ring stages are deferred until the epilogue has read that one
+//     too (the stages are released after those).
 //
 // Kernel structure (persistent, clusters of 2 CTAs = one SM pair, 192 threads each):
-//   warp 0  TMA producer (both CTAs): streams 64-wide K slices of its 128 rows
-//           of H and of its bn/2 of the tile's bn W rows into a 6-stage ring;
-//           both CTAs' copies complete on the LEADER's stage barrier;
-//   warp 1  TMEM allocation (both CTAs, 512 columns = two 256-column fp32
-//           accumulators) and, in the leader only, the MMA issuer:
-//           4 x (M256 Nbn K16) per stage, committing stage release and
-//           accumulator-ready to both CTAs (multicast);
+//   warp 0  TMA producer (both CTAs): per K slice, its 128 rows of H and its
+//           bn/2 of the (one or two) tiles' W rows into the ring; both CTAs'
+//           copies complete on the LEADER's stage barrier;
+//   warp 1  TMEM allocation (both CTAs, all 512 columns) and, in the leader
+//           only, the MMA issuer: 4 x (M256 Nbn K16) per stage and tile,
+//           committing stage release and accumulator-ready to both CTAs
+//           (multicast);
 //   warps 2-5 epilogue (both CTAs): one thread per row (TMEM lane); online
-//           softmax over a tile's bn columns while the MMAs of the next tile
-//           fill the other accumulator, then release the accumulator to the
-//           leader's MMA warp (8 arrivals per tile).
+//           softmax over a tile's columns, then release of the accumulator to
+//           the leader's MMA warp (8 arrivals per accumulator use).
 // Work split: see ScoreArgs in internal.h.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA raises an
@@ -46,20 +59,122 @@ namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint16_t kBothCtas = 0x3;
-constexpr int kPrefetchSlices = 16;  // K slices of the first tile prefetched into L2 before the grid wait
+constexpr int kPrefetchSlices = 4;   // K slices of the first W tile prefetched into L2 before the grid wait
+constexpr int kTmemLoadsPerWait = 1;  // 32-column TMEM loads in flight per tcgen05.wait::ld in the epilogue (2 measured slower)
 
 struct alignas(8) Barriers {
-    uint64_t full[kStages];   // leader: both CTAs' copies of a stage landed
-    uint64_t empty[kStages];  // both: the stage's MMAs are done (multicast commit)
-    uint64_t tmem_full[2];    // both: accumulator i holds a finished tile (multicast commit)
-    uint64_t tmem_empty[2];   // leader: all 8 epilogue warps of the pair have read accumulator i
-    uint64_t mma_done;        // leader: every MMA issued has completed
+    uint64_t full[kMaxStages];   // leader: both CTAs' copies of a stage landed
+    uint64_t empty[kMaxStages];  // both: the stage's MMAs are done (multicast commit)
+    uint64_t tmem_full[2];       // both: accumulator i holds a finished tile (multicast commit)
+    uint64_t tmem_empty[2];      // leader: all 8 epilogue warps of the pair have read accumulator i
+    uint64_t mma_done;           // leader: every MMA issued has completed
     uint32_t tmem_base;
     int32_t abort;
 };
 static_assert(sizeof(Barriers) <= 256, "barrier block must fit its reserve");
 
+// Running softmax state of one row (one thread), across all of a pair's tiles of that row.
+struct RowState {
+    float m, s0, s1, s2, s3, tlog;
+    float u0, u1, u2, u3;  // entropy variant: sum of exp(l - m) (l - m) log2(e)
+    int32_t am;
+};
+
+// Fold 32 consecutive logits x (columns v .. v + 31; those at or past cvalid are not logits) into the row
+// state: online max with rescaling, four partial sums of 2^((l - m) log2 e), argmax (an earlier column
+// keeps it on ties), and the target's logit when it lies among them.
 template <bool kEntropy>
+__device__ __forceinline__ void fold32(RowState &r, float (&x)[32], int v, int cvalid, int tgt)
+{
+    if (cvalid < 32) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j >= cvalid)
+                x[j] = -INFINITY;  // past V (TMA zero fill) or past the tile (another tile's columns)
+    }
+    float cm = x[0];
+#pragma unroll
+    for (int j = 1; j < 32; ++j)
+        cm = fmaxf(cm, x[j]);
+    if (cm > r.m) {  // strict: an earlier column keeps the argmax on ties
+        int j0 = 31;
+#pragma unroll
+        for (int j = 31; j >= 0; --j)
+            if (x[j] == cm)
+                j0 = j;
+        r.am = v + j0;
+        const float scale = ptx::ex2((r.m - cm) * kLog2e);
+        if (kEntropy && r.m != -INFINITY) {  // u' = scale * (u + (m - cm) log2(e) * s)
+            const float dl = (r.m - cm) * kLog2e;
+            r.u0 = scale * fmaf(dl, r.s0, r.u0);
+            r.u1 = scale * fmaf(dl, r.s1, r.u1);
+            r.u2 = scale * fmaf(dl, r.s2, r.u2);
+            r.u3 = scale * fmaf(dl, r.s3, r.u3);
+        }
+        r.s0 *= scale;
+        r.s1 *= scale;
+        r.s2 *= scale;
+        r.s3 *= scale;
+        r.m = cm;
+    }
+    const float mb2 = r.m * kLog2e;
+    if (!kEntropy) {
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+            r.s0 += ptx::ex2(fmaf(x[j + 0], kLog2e, -mb2));
+            r.s1 += ptx::ex2(fmaf(x[j + 1], kLog2e, -mb2));
+            r.s2 += ptx::ex2(fmaf(x[j + 2], kLog2e, -mb2));
+            r.s3 += ptx::ex2(fmaf(x[j + 3], kLog2e, -mb2));
+        }
+    } else {
+        // t = (l - m) log2(e), kept finite (masked columns are -inf; 2^-200 is 0 in fp32 anyway)
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+            const float t0 = fmaxf(fmaf(x[j + 0], kLog2e, -mb2), -200.f);
+            const float t1 = fmaxf(fmaf(x[j + 1], kLog2e, -mb2), -200.f);
+            const float t2 = fmaxf(fmaf(x[j + 2], kLog2e, -mb2), -200.f);
+            const float t3 = fmaxf(fmaf(x[j + 3], kLog2e, -mb2), -200.f);
+            const float e0 = ptx::ex2(t0), e1 = ptx::ex2(t1), e2 = ptx::ex2(t2), e3 = ptx::ex2(t3);
+            r.s0 += e0;
+            r.s1 += e1;
+            r.s2 += e2;
+            r.s3 += e3;
+            r.u0 = fmaf(e0, t0, r.u0);
+            r.u1 = fmaf(e1, t1, r.u1);
+            r.u2 = fmaf(e2, t2, r.u2);
+            r.u3 = fmaf(e3, t3, r.u3);
+        }
+    }
+    const int tj = tgt - v;
+    if ((unsigned)tj < 32u) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            r.tlog = (j == tj) ? x[j] : r.tlog;
+    }
+}
+
+// Fold the nvalid first columns of one accumulator (this warp's 32 TMEM lanes from tbase), vocabulary
+// ids v0 ..; kTmemLoadsPerWait 32-column loads in flight per wait.
+template <bool kEntropy>
+__device__ __forceinline__ void fold_tile(RowState &r, uint32_t tbase, int v0, int nvalid, int tgt)
+{
+#pragma unroll 1
+    for (int c = 0; c * 32 < nvalid; c += kTmemLoadsPerWait) {
+        float x[kTmemLoadsPerWait][32];
+#pragma unroll
+        for (int i = 0; i < kTmemLoadsPerWait; ++i)
+            if (i == 0 || (c + i) * 32 < nvalid)  // warp-uniform
+                ptx::tmem_ld_32x32b_x32(tbase + (uint32_t)((c + i) * 32), x[i]);
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < kTmemLoadsPerWait; ++i)
+            if (i == 0 || (c + i) * 32 < nvalid)
+                fold32<kEntropy>(r, x[i], v0 + (c + i) * 32, nvalid - (c + i) * 32, tgt);
+    }
+}
+
+// kTwo: two-tile passes (ScoreArgs::two == 1), else single tiles.
+template <bool kEntropy, bool kTwo>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW,
                  const ScoreArgs a)
@@ -67,7 +182,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_u32(smem_raw);
     const uint32_t ring = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-B alignment
-    Barriers *bars = reinterpret_cast<Barriers *>(smem_raw + (ring - raw) + kRingBytes);
+    Barriers *bars = reinterpret_cast<Barriers *>(smem_raw + (ring - raw) + (uint32_t)a.stages * a.stage_bytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = ptx::cluster_ctarank();  // 0: leader (issues the MMAs), 1: peer
     const bool leader = rank == 0;
@@ -76,8 +191,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     if (tl && threadIdx.x == 0)
         tl[0] = ptx::globaltimer_ns();
 
-    auto sA = [&](int s) { return ring + (uint32_t)s * (kStageBytesA + kStageBytesB); };
-    auto sB = [&](int s) { return sA(s) + kStageBytesA; };
+    const int S = a.stages;
+    const uint32_t wb = stage_bytes_w(a.bn);
+    auto sA = [&](int s) { return ring + (uint32_t)s * a.stage_bytes; };
+    auto sB = [&](int s, int t) { return sA(s) + kStageBytesA + (uint32_t)t * wb; };
     auto full = [&](int s) { return ptx::smem_u32(&bars->full[s]); };
     auto empty = [&](int s) { return ptx::smem_u32(&bars->empty[s]); };
     auto tfull = [&](int i) { return ptx::smem_u32(&bars->tmem_full[i]); };
@@ -86,7 +203,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
     // Set-up that touches no global memory overlaps the previous kernel (programmatic launch).
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < S; ++s) {
             ptx::mbar_init(full(s), 1);
             ptx::mbar_init(empty(s), 1);
         }
@@ -120,11 +237,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     // Programmatic launch: everything above overlapped the grid before us.  Whatever that grid is (the
     // previous WINO call's finish kernel, or a kernel of the caller's that wrote H), its writes are only
     // visible after griddepcontrol.wait, so every role waits before its first global access; the producer
-    // first prefetches the start of its first tile into L2, which is safe before the wait (L2 is coherent).
+    // first prefetches the start of its first W tile into L2, which is safe before the wait (L2 is coherent).
     ptx::grid_dep_launch_dependents();
 
     const int grp = pair % a.n_groups;  // 256-row blocks grp, grp + n_groups, ...
     const int col = pair / a.n_groups;  // vocabulary tiles col, col + G, ...
+    const int vstep = kTwo ? 2 * a.G : a.G;  // tiles per item: 1, or 2 (col + 2jG and col + (2j+1)G)
 
     if (warp >= 2 || !tmem_ok) {
         ptx::grid_dep_wait();
@@ -141,26 +259,23 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer (both CTAs)
         const int half_bn = a.bn >> 1;  // W rows each CTA stages per tile
-        if (lane == 0 && grp < a.n_mb && col < a.n_vt) {
-            const int n_pre = min(a.n_kb, kPrefetchSlices);
-            for (int kb = 0; kb < n_pre; ++kb) {
+        if (lane == 0 && grp < a.n_mb)
+            for (int kb = 0; kb < min(a.n_kb, kPrefetchSlices); ++kb)
                 ptx::tma_prefetch_2d(&tmW, kb * kBK, col * a.bn + (int)rank * half_bn);
-                ptx::tma_prefetch_2d(&tmH, kb * kBK, grp * kPairM + (int)rank * kBM);
-            }
-        }
         ptx::grid_dep_wait();
-        const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every vocabulary tile
+        const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every item
         const uint64_t pol_w = ptx::policy_evict_normal();  // W is shared by the row-block groups
         int stage = 0;
         uint32_t phase = 0;
-        int32_t issued_parity[kStages];
-        for (int s = 0; s < kStages; ++s)
+        int32_t issued_parity[kMaxStages];
+        for (int s = 0; s < kMaxStages; ++s)
             issued_parity[s] = -1;
         bool aborted = false;
-        const uint32_t stage_tx = 2 * (kStageBytesA + (uint32_t)half_bn * (kBK * 2));  // both CTAs' copies
         bool first = true;
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-            for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
+            for (int vt = col; vt < a.n_vt && !aborted; vt += vstep) {
+                const bool two = kTwo && vt + a.G < a.n_vt;
+                const uint32_t stage_tx = 2u * (kStageBytesA + (two ? 2u : 1u) * wb);  // both CTAs' copies
                 for (int kb = 0; kb < a.n_kb; ++kb) {
                     int ok = 1;
                     if (lane == 0)
@@ -175,15 +290,18 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         if (leader)
                             ptx::mbar_arrive_expect_tx(full(stage), stage_tx);
                         ptx::tma_load_2d_pair(sA(stage), &tmH, bar, kb * kBK, mb * kPairM + (int)rank * kBM, pol_h);
-                        ptx::tma_load_2d_pair(sB(stage), &tmW, bar, kb * kBK, vt * a.bn + (int)rank * half_bn,
+                        ptx::tma_load_2d_pair(sB(stage, 0), &tmW, bar, kb * kBK, vt * a.bn + (int)rank * half_bn,
                                               pol_w);
+                        if (two)
+                            ptx::tma_load_2d_pair(sB(stage, 1), &tmW, bar, kb * kBK,
+                                                  (vt + a.G) * a.bn + (int)rank * half_bn, pol_w);
                         if (tl && first)
                             tl[2] = ptx::globaltimer_ns();
                         first = false;
                     }
                     __syncwarp();
                     issued_parity[stage] = (int32_t)phase;
-                    if (++stage == kStages) {
+                    if (++stage == S) {
                         stage = 0;
                         phase ^= 1u;
                     }
@@ -192,7 +310,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         }
         if (aborted && leader && lane == 0) {
             // Let every copy already issued (by either CTA) land before the pair's shared memory goes away.
-            for (int s = 0; s < kStages; ++s)
+            for (int s = 0; s < S; ++s)
                 if (issued_parity[s] >= 0)
                     wait_drain(full(s), (uint32_t)issued_parity[s]);
         }
@@ -204,23 +322,38 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             int tiles = 0;
             int stage = 0;
             uint32_t phase = 0;
-            int acc = 0;
-            uint32_t acc_phase = 0;
+            int item = 0;  // items issued so far
             bool aborted = false;
+            auto wait_acc_free = [&](int i, uint32_t uses) -> bool {  // the epilogue has read use uses-1 of acc i
+                int ok = 1;
+                if (lane == 0)
+                    ok = wait_bounded<true>(tempty(i), (uses & 1u) ^ 1u, &bars->abort);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                ptx::tc_fence_after();
+                return ok != 0;
+            };
+            auto issue = [&](int acc, int s, int tile, int kb) {  // 4 x K16 of one tile from stage s
+                const uint64_t da = ptx::sdesc_kmajor_sw128(sA(s));
+                const uint64_t db = ptx::sdesc_kmajor_sw128(sB(s, tile));
+#pragma unroll
+                for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
+                    ptx::mma_bf16_pair(tmem + (uint32_t)acc * kBN, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
+            };
             for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-                for (int vt = col; vt < a.n_vt && !aborted; vt += a.G) {
-                    int ok = 1;
-                    if (lane == 0)
-                        ok = wait_bounded<true>(tempty(acc), acc_phase ^ 1u, &bars->abort);
-                    ok = __shfl_sync(0xffffffffu, ok, 0);
-                    if (!ok) {
+                for (int vt = col; vt < a.n_vt && !aborted; vt += vstep, ++item) {
+                    const bool two = kTwo && vt + a.G < a.n_vt;
+                    // single tiles: item i uses accumulator i & 1 for the (i >> 1)-th time;
+                    // passes: item i uses both accumulators for the i-th time
+                    const int acc0 = kTwo ? 0 : (item & 1);
+                    const uint32_t uses0 = kTwo ? (uint32_t)item : (uint32_t)(item >> 1);
+                    if (!wait_acc_free(acc0, uses0)) {
                         aborted = true;
                         break;
                     }
-                    ptx::tc_fence_after();
-                    const uint32_t d_tmem = tmem + (uint32_t)(acc * kBN);
+                    const int defer = two ? min(S, a.n_kb) : 0;  // stages whose second-tile MMAs wait
+                    const int s0 = stage;
                     for (int kb = 0; kb < a.n_kb; ++kb) {
-                        ok = 1;
+                        int ok = 1;
                         if (lane == 0)
                             ok = wait_bounded(full(stage), phase, &bars->abort);
                         ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -229,30 +362,41 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                             break;
                         }
                         ptx::tc_fence_after();
-                        if (lane == 0) {
-                            const uint64_t da = ptx::sdesc_kmajor_sw128(sA(stage));
-                            const uint64_t db = ptx::sdesc_kmajor_sw128(sB(stage));
-#pragma unroll
-                            for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
-                                ptx::mma_bf16_pair(d_tmem, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
+                        if (lane == 0)
+                            issue(acc0, stage, 0, kb);
+                        if (kb < defer) {
+                            if (kb == defer - 1) {  // the second accumulator is needed now
+                                if (!wait_acc_free(1, (uint32_t)item)) {
+                                    aborted = true;
+                                    break;
+                                }
+                                if (lane == 0)
+                                    for (int j = 0; j < defer; ++j) {
+                                        const int sj = (s0 + j) % S;
+                                        issue(1, sj, 1, j);
+                                        ptx::mma_commit_pair_multicast(empty(sj), kBothCtas);
+                                    }
+                            }
+                        } else if (lane == 0) {
+                            if (two)
+                                issue(1, stage, 1, kb);
                             ptx::mma_commit_pair_multicast(empty(stage), kBothCtas);
                         }
                         __syncwarp();
-                        if (++stage == kStages) {
+                        if (++stage == S) {
                             stage = 0;
                             phase ^= 1u;
                         }
                     }
                     if (aborted)
                         break;
-                    if (lane == 0)
-                        ptx::mma_commit_pair_multicast(tfull(acc), kBothCtas);
-                    __syncwarp();
-                    ++tiles;
-                    if (++acc == 2) {
-                        acc = 0;
-                        acc_phase ^= 1u;
+                    if (lane == 0) {
+                        ptx::mma_commit_pair_multicast(tfull(acc0), kBothCtas);
+                        if (kTwo)  // the epilogue waits for both accumulators of every pass
+                            ptx::mma_commit_pair_multicast(tfull(1), kBothCtas);
                     }
+                    __syncwarp();
+                    tiles += two ? 2 : 1;
                 }
             }
             // No MMA may still be writing either CTA's TMEM when it is released.
@@ -269,116 +413,51 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     } else {
         // ------------------------------------------------------------ epilogue (warps 2..5, both CTAs)
         const int q = warp & 3;  // this warp may only read TMEM lanes [32q, 32q + 32)
-        int acc = 0;
-        uint32_t acc_phase = 0;
+        const uint32_t lanes = tmem + ((uint32_t)(q * 32) << 16);
+        int item = 0;
         bool aborted = false;
+        auto take = [&](int i, uint32_t uses) -> bool {  // wait for use `uses` of accumulator i
+            int ok = 1;
+            if (lane == 0)
+                ok = wait_bounded(tfull(i), uses & 1u, &bars->abort);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            ptx::tc_fence_after();
+            return ok != 0;
+        };
+        auto release = [&](int i) {  // accumulator i fully read by this warp: tell the leader's MMA warp
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                ptx::mbar_arrive_cluster(ptx::mapa(tempty(i), 0));
+        };
         for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
             const int64_t row = (int64_t)mb * kPairM + (int)rank * kBM + q * 32 + lane;
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
-            float m = -INFINITY, s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f, tlog = -INFINITY;
-            float u0 = 0.f, u1 = 0.f, u2 = 0.f, u3 = 0.f;  // entropy variant
-            int32_t am = 0;
-            for (int vt = col; vt < a.n_vt; vt += a.G) {
-                const int32_t v0 = vt * a.bn;
-                const int nvalid = min(a.bn, a.V - v0);
-                int ok = 1;
-                if (lane == 0)
-                    ok = wait_bounded(tfull(acc), acc_phase, &bars->abort);
-                ok = __shfl_sync(0xffffffffu, ok, 0);
-                if (!ok) {
+            RowState r{-INFINITY, 0.f, 0.f, 0.f, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0};
+            for (int vt = col; vt < a.n_vt; vt += vstep, ++item) {
+                const int acc0 = kTwo ? 0 : (item & 1);
+                const uint32_t uses0 = kTwo ? (uint32_t)item : (uint32_t)(item >> 1);
+                if (!take(acc0, uses0)) {
                     aborted = true;
                     break;
                 }
-                ptx::tc_fence_after();
-                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
-#pragma unroll 1
-                for (int c = 0; c < kBN / 32; ++c) {
-                    const int cvalid = nvalid - c * 32;  // warp-uniform; columns past the tile are masked
-                    if (cvalid <= 0)
+                fold_tile<kEntropy>(r, lanes + (uint32_t)acc0 * kBN, vt * a.bn, min(a.bn, a.V - vt * a.bn), tgt);
+                release(acc0);
+                if (kTwo) {
+                    if (!take(1, (uint32_t)item)) {
+                        aborted = true;
                         break;
-                    float x[32];
-                    ptx::tmem_ld_32x32b_x32(tbase + (uint32_t)(c * 32), x);
-                    ptx::tmem_ld_wait();
-                    if (cvalid < 32) {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (j >= cvalid)
-                                x[j] = -INFINITY;  // past V (TMA zero fill) or past the tile (another tile's columns)
                     }
-                    float cm = x[0];
-#pragma unroll
-                    for (int j = 1; j < 32; ++j)
-                        cm = fmaxf(cm, x[j]);
-                    if (cm > m) {  // strict: an earlier column keeps the argmax on ties
-                        int j0 = 31;
-#pragma unroll
-                        for (int j = 31; j >= 0; --j)
-                            if (x[j] == cm)
-                                j0 = j;
-                        am = v0 + c * 32 + j0;
-                        const float scale = ptx::ex2((m - cm) * kLog2e);
-                        if (kEntropy && m != -INFINITY) {  // u' = scale * (u + (m - cm) log2(e) * s)
-                            const float dl = (m - cm) * kLog2e;
-                            u0 = scale * fmaf(dl, s0, u0);
-                            u1 = scale * fmaf(dl, s1, u1);
-                            u2 = scale * fmaf(dl, s2, u2);
-                            u3 = scale * fmaf(dl, s3, u3);
-                        }
-                        s0 *= scale;
-                        s1 *= scale;
-                        s2 *= scale;
-                        s3 *= scale;
-                        m = cm;
-                    }
-                    const float mb2 = m * kLog2e;
-                    if (!kEntropy) {
-#pragma unroll
-                        for (int j = 0; j < 32; j += 4) {
-                            s0 += ptx::ex2(fmaf(x[j + 0], kLog2e, -mb2));
-                            s1 += ptx::ex2(fmaf(x[j + 1], kLog2e, -mb2));
-                            s2 += ptx::ex2(fmaf(x[j + 2], kLog2e, -mb2));
-                            s3 += ptx::ex2(fmaf(x[j + 3], kLog2e, -mb2));
-                        }
-                    } else {
-                        // t = (l - m) log2(e), kept finite (masked columns are -inf; 2^-200 is 0 in fp32 anyway)
-#pragma unroll
-                        for (int j = 0; j < 32; j += 4) {
-                            const float t0 = fmaxf(fmaf(x[j + 0], kLog2e, -mb2), -200.f);
-                            const float t1 = fmaxf(fmaf(x[j + 1], kLog2e, -mb2), -200.f);
-                            const float t2 = fmaxf(fmaf(x[j + 2], kLog2e, -mb2), -200.f);
-                            const float t3 = fmaxf(fmaf(x[j + 3], kLog2e, -mb2), -200.f);
-                            const float e0 = ptx::ex2(t0), e1 = ptx::ex2(t1), e2 = ptx::ex2(t2), e3 = ptx::ex2(t3);
-                            s0 += e0;
-                            s1 += e1;
-                            s2 += e2;
-                            s3 += e3;
-                            u0 = fmaf(e0, t0, u0);
-                            u1 = fmaf(e1, t1, u1);
-                            u2 = fmaf(e2, t2, u2);
-                            u3 = fmaf(e3, t3, u3);
-                        }
-                    }
-                    const int tj = tgt - (v0 + c * 32);
-                    if ((unsigned)tj < 32u) {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            tlog = (j == tj) ? x[j] : tlog;
-                    }
-                }
-                // Accumulator fully read by this warp: tell the leader's MMA warp.
-                ptx::tc_fence_before();
-                __syncwarp();
-                if (lane == 0)
-                    ptx::mbar_arrive_cluster(ptx::mapa(tempty(acc), 0));
-                if (++acc == 2) {
-                    acc = 0;
-                    acc_phase ^= 1u;
+                    const int vt1 = vt + a.G;
+                    if (vt1 < a.n_vt)
+                        fold_tile<kEntropy>(r, lanes + kBN, vt1 * a.bn, min(a.bn, a.V - vt1 * a.bn), tgt);
+                    release(1);
                 }
             }
             if (!aborted && row < a.N) {
-                a.part[row * a.G + col] = make_float4(m, (s0 + s1) + (s2 + s3), __int_as_float(am), tlog);
+                a.part[row * a.G + col] = make_float4(r.m, (r.s0 + r.s1) + (r.s2 + r.s3), __int_as_float(r.am), r.tlog);
                 if (kEntropy)
-                    a.part_u[row * a.G + col] = (u0 + u1) + (u2 + u3);
+                    a.part_u[row * a.G + col] = (r.u0 + r.u1) + (r.u2 + r.u3);
             }
         }
         if (tl && !leader && warp == 2 && lane == 0)
@@ -408,14 +487,23 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
 }  // namespace
 
-// Choose the tile width bn and the number of row-block groups: fewest vocabulary columns on the busiest
-// pair (tiles x (bn + a per-tile overhead)), then the widest tile, then fewest passes over W (more groups).
-// A width below kBN pays when the vocabulary then splits evenly over the pairs: V = 126464 on 76 pairs is
-// 494 tiles of 256 (7 on the busiest pair, 6.5 on average) but 527 tiles of 240 (7 on the busiest pair).
+// Choose the mode, the tile width bn and the number of row-block groups.  One 256-row block is bound by the
+// W stream from HBM: single tiles (the most bytes in flight).  More rows are tensor-bound: two-tile passes
+// (fewer bytes delivered per MMA).  Then: fewest vocabulary columns on the busiest pair plus a per-tile or
+// per-pass overhead, the widest tile, fewest passes over W (more groups).  A width below kBN pays when the
+// vocabulary then splits evenly over the pairs: V = 126464 on 76 pairs is 494 tiles of 256 (7 on the
+// busiest pair, 6.5 on average) but 527 tiles of 240 (7 on 71 pairs).
+#ifndef WINO_PASS_MIN_ROW_BLOCKS
+#define WINO_PASS_MIN_ROW_BLOCKS 2  // compile-time tuning: fewest 256-row blocks that use two-tile passes
+#endif
+constexpr int32_t kPassMinRowBlocks = WINO_PASS_MIN_ROW_BLOCKS;
+
 ScoreSchedule score_schedule(int32_t n_mb, int64_t V, int max_units, int32_t records_cap)
 {
-    constexpr int64_t kTileOverheadCols = 16;  // H re-read and accumulator hand-over per tile, in columns
-    ScoreSchedule best{kBN, (int32_t)((V + kBN - 1) / kBN), 1, 1};
+    constexpr int64_t kTileOverheadCols = 16;  // single tiles: H re-staged per tile, in columns
+    constexpr int64_t kPassOverheadCols = 32;  // passes: the epilogue the next pass partly waits for
+    const int32_t two = n_mb >= kPassMinRowBlocks ? 1 : 0;
+    ScoreSchedule best{kBN, (int32_t)((V + kBN - 1) / kBN), 1, 1, two, 2, 0};
     int64_t best_cost = -1;
     const int32_t top = n_mb < max_units ? n_mb : max_units;
     for (int32_t bn = kBN; bn >= kMinBN; bn -= 16) {
@@ -426,25 +514,33 @@ ScoreSchedule score_schedule(int32_t n_mb, int64_t V, int max_units, int32_t rec
             g = g < records_cap ? g : records_cap;
             g = g < kMaxRecordsPerRow ? g : kMaxRecordsPerRow;
             g = g < 1 ? 1 : g;
-            const int64_t rounds = (int64_t)((n_mb + groups - 1) / groups) * ((n_vt + g - 1) / g);
-            const int64_t cost = rounds * (bn + kTileOverheadCols);
+            const int64_t tiles = (n_vt + g - 1) / g;  // on the busiest pair, per row block
+            const int64_t per_mb = two ? tiles * bn + ((tiles + 1) / 2) * kPassOverheadCols
+                                       : tiles * (bn + kTileOverheadCols);
+            const int64_t cost = (int64_t)((n_mb + groups - 1) / groups) * per_mb;
             if (best_cost < 0 || cost < best_cost) {
                 best_cost = cost;
-                best = ScoreSchedule{bn, (int32_t)n_vt, groups, (int32_t)g};
+                best.bn = bn;
+                best.n_vt = (int32_t)n_vt;
+                best.n_groups = groups;
+                best.G = (int32_t)g;
             }
         }
     }
+    best.stage_bytes = kStageBytesA + (uint32_t)(1 + two) * stage_bytes_w(best.bn);
+    const uint32_t fit = kRingCapacity / best.stage_bytes;
+    best.stages = (int32_t)(fit < (uint32_t)kMaxStages ? fit : (uint32_t)kMaxStages);
     return best;
 }
 
 namespace {
 
-cudaLaunchConfig_t score_config(unsigned grid, cudaStream_t stream, cudaLaunchAttribute (&attr)[2])
+cudaLaunchConfig_t score_config(unsigned grid, uint32_t smem, cudaStream_t stream, cudaLaunchAttribute (&attr)[2])
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kScoreThreads);
-    cfg.dynamicSmemBytes = kScoreSmemBytes;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
@@ -468,16 +564,17 @@ int configure_device()
         return -1;
     std::lock_guard<std::mutex> g(mu);
     if (!done[dev]) {
-        if (cudaFuncSetAttribute(score_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kScoreSmemBytes) != cudaSuccess ||
-            cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kScoreSmemBytes) != cudaSuccess)
-            return -1;
+        for (auto *k : {score_kernel<false, false>, score_kernel<false, true>, score_kernel<true, false>,
+                        score_kernel<true, true>})
+            if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScoreSmemMax) !=
+                cudaSuccess)
+                return -1;
         cudaLaunchAttribute attr[2];
-        cudaLaunchConfig_t cfg = score_config(2, nullptr, attr);
+        // Any launch's shared memory exceeds half an SM's, so one CTA per SM whatever the ring size.
+        cudaLaunchConfig_t cfg = score_config(2, kScoreSmemMax, nullptr, attr);
         cfg.numAttrs = 1;  // the cluster shape is what matters for the occupancy query
         int clusters = 0;
-        if (cudaOccupancyMaxActiveClusters(&clusters, score_kernel<false>, &cfg) != cudaSuccess || clusters < 1)
+        if (cudaOccupancyMaxActiveClusters(&clusters, score_kernel<false, true>, &cfg) != cudaSuccess || clusters < 1)
             return -1;
         pairs[dev] = clusters;
         done[dev] = true;
@@ -495,9 +592,13 @@ cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const S
     if (configure_device() < 1)
         return cudaErrorUnknown;
     cudaLaunchAttribute attr[2];
-    cudaLaunchConfig_t cfg = score_config((unsigned)(2 * a.n_groups * a.G), stream, attr);
-    return entropy ? cudaLaunchKernelEx(&cfg, score_kernel<true>, tmH, tmW, a)
-                   : cudaLaunchKernelEx(&cfg, score_kernel<false>, tmH, tmW, a);
+    cudaLaunchConfig_t cfg = score_config((unsigned)(2 * a.n_groups * a.G),
+                                          kSmemOverhead + (uint32_t)a.stages * a.stage_bytes, stream, attr);
+    if (entropy)
+        return a.two ? cudaLaunchKernelEx(&cfg, score_kernel<true, true>, tmH, tmW, a)
+                     : cudaLaunchKernelEx(&cfg, score_kernel<true, false>, tmH, tmW, a);
+    return a.two ? cudaLaunchKernelEx(&cfg, score_kernel<false, true>, tmH, tmW, a)
+                 : cudaLaunchKernelEx(&cfg, score_kernel<false, false>, tmH, tmW, a);
 }
 
 }  // namespace wino

@@ -246,6 +246,9 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     a.n_vt = sch.n_vt;
     a.n_kb = (int32_t)((d + kBK - 1) / kBK);
     a.bn = sch.bn;
+    a.two = sch.two;
+    a.stages = sch.stages;
+    a.stage_bytes = sch.stage_bytes;
     a.n_groups = sch.n_groups;
     a.G = sch.G;
     a.ts = ts;
@@ -530,6 +533,8 @@ int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan)
     plan[3] = sch.n_groups;
     plan[4] = sch.G;
     plan[5] = 2 * sch.n_groups * sch.G;
+    plan[6] = sch.two;
+    plan[7] = sch.stages;
     return WINO_OK;
 }
 
