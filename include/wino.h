@@ -321,10 +321,14 @@ WINO_API int wino_profile_end(double *score_ms_total, int *score_launches);
  * tensor memory), [2] first tensor copy issued, [3] wait for the previous
  * kernel done, [4] last MMA completed (leader CTA of a pair) or last tile
  * read (the other CTA), [5] all roles done, [6] exit; and [7] = SM id << 32
- * | tiles of the CTA pair (leader CTA).  A launch with more CTAs than
- * ctas_per_launch writes nothing.  buf is a device buffer of
- * n_launches * ctas_per_launch * 8 uint64 owned by the caller; end returns how
- * many launches were counted.  One timeline per process at a time.
+ * | tiles of the CTA pair (leader CTA).  Stamps [0], [1], [2], [5] and [6]
+ * come from one thread and are ordered; [3] and [4] come from other warps,
+ * whose %globaltimer readings were seen to disagree with it by up to a few
+ * microseconds, so compare those only with each other or across CTAs.
+ * A launch with more CTAs than ctas_per_launch writes nothing.  buf is a
+ * device buffer of n_launches * ctas_per_launch * 8 uint64 owned by the
+ * caller; end returns how many launches were counted.  One timeline per
+ * process at a time.
  */
 WINO_API int wino_timeline_begin(uint64_t *buf, int64_t n_launches, int64_t ctas_per_launch);
 WINO_API int wino_timeline_end(int64_t *launches);
