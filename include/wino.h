@@ -346,6 +346,16 @@ WINO_API int wino_timeline_end(int64_t *launches);
 WINO_API int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan);
 
 /*
+ * The same work split for a device with sm_count SMs of which max_pairs CTA
+ * pairs of the score kernel can be resident (152 and 76 on a GB300), without
+ * touching any device (capacity planning, host-side tests).  plan (host
+ * int32[10]) receives the eight fields of wino_score_plan, then the bytes of
+ * one ring stage and the partial records the workspace holds per row.
+ */
+WINO_API int wino_score_plan_host(int64_t N, int64_t d, int64_t V, int32_t sm_count, int32_t max_pairs,
+                                  int32_t *plan);
+
+/*
  * Self-test of the failure path (device-side timeout handling; the paper has
  * no counterpart).  Enqueues one small kernel that waits, with the library's
  * bounded wait shortened to limit_ns (1 us .. 1 s), on a barrier nothing

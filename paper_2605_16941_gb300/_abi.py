@@ -34,7 +34,7 @@ WINO_OPT_COMPACT = 4
 EXPORTS = ("wino_workspace_size", "wino_workspace_size_step", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
            "wino_selftest_wait_timeout", "wino_status_string", "wino_version", "wino_decode", "wino_timeline_begin",
-           "wino_timeline_end", "wino_score_plan")
+           "wino_timeline_end", "wino_score_plan", "wino_score_plan_host")
 
 # 64-bit words per CTA in a score-kernel timeline (wino_timeline_begin)
 TIMELINE_WORDS = 8
@@ -96,6 +96,8 @@ def lib() -> C.CDLL:
         L.wino_profile_begin.argtypes = [C.c_int]
         L.wino_profile_end.restype = C.c_int
         L.wino_profile_end.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_int)]
+        L.wino_score_plan_host.restype = C.c_int
+        L.wino_score_plan_host.argtypes = [i64, i64, i64, C.c_int32, C.c_int32, C.POINTER(C.c_int32)]
         L.wino_score_plan.restype = C.c_int
         L.wino_score_plan.argtypes = [i64, i64, i64, C.POINTER(C.c_int32)]
         L.wino_timeline_begin.restype = C.c_int
@@ -279,6 +281,15 @@ def wino_score_plan(N: int, d: int, V: int) -> dict:
     out = (C.c_int32 * 8)()
     _check(lib().wino_score_plan(int(N), int(d), int(V), out), "wino_score_plan")
     return dict(zip(("bn", "n_vt", "n_mb", "n_groups", "G", "ctas", "two", "stages"), list(out)))
+
+
+def wino_score_plan_host(N: int, d: int, V: int, sm_count: int = 152, max_pairs: int = 76) -> dict:
+    """The score kernel's work split for a device with sm_count SMs and max_pairs resident pairs (no device)."""
+    out = (C.c_int32 * 10)()
+    _check(lib().wino_score_plan_host(int(N), int(d), int(V), int(sm_count), int(max_pairs), out),
+           "wino_score_plan_host")
+    return dict(zip(("bn", "n_vt", "n_mb", "n_groups", "G", "ctas", "two", "stages", "stage_bytes",
+                     "records_per_row"), list(out)))
 
 
 def wino_timeline_begin(buf, n_launches: int, ctas_per_launch: int) -> None:

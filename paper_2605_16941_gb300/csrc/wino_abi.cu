@@ -511,6 +511,28 @@ int wino_read_device_status(const void *ws, void *stream, int *device_status)
     return WINO_OK;
 }
 
+int wino_score_plan_host(int64_t N, int64_t d, int64_t V, int32_t sm_count, int32_t max_pairs, int32_t *plan)
+{
+    if (!plan || sm_count < 2 || max_pairs < 1)
+        return WINO_ERR_ARG;
+    if (!shape_ok(N, d, V))
+        return WINO_ERR_SHAPE;
+    const int32_t n_mb = (int32_t)((N + kPairM - 1) / kPairM);
+    const ScoreSchedule sch =
+        score_schedule(n_mb, V, std::min(max_pairs, sm_count / 2), (int32_t)records_per_row(V));
+    plan[0] = sch.bn;
+    plan[1] = sch.n_vt;
+    plan[2] = n_mb;
+    plan[3] = sch.n_groups;
+    plan[4] = sch.G;
+    plan[5] = 2 * sch.n_groups * sch.G;
+    plan[6] = sch.two;
+    plan[7] = sch.stages;
+    plan[8] = (int32_t)sch.stage_bytes;
+    plan[9] = (int32_t)records_per_row(V);
+    return WINO_OK;
+}
+
 int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan)
 {
     if (!plan)
