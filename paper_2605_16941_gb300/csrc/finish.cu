@@ -16,7 +16,7 @@
 // score kernel and it waits (griddepcontrol.wait) for the score kernel's
 // results before touching them; it lets the next call's kernels launch at once
 // (they only read H and W before their own griddepcontrol.wait).  The last of
-// its CTAs publishes the call's status word (see StatusWords).
+// its CTAs publishes the call's status (see StatusWords).
 //
 // draft_verify_kernel: Eq. 4 alone from caller-supplied statistics
 // (wino_draft_verify), one CTA per sequence.

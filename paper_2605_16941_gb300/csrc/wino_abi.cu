@@ -3,7 +3,7 @@
 // Host side only: argument and shape checks, workspace layout, TMA tensor-map
 // encoding (cached), and kernel launches on the caller's stream.  No entry
 // point allocates device memory or synchronises, except
-// wino_read_device_status, which reads one status word back.
+// wino_read_device_status, which reads the status words back.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
