@@ -103,3 +103,15 @@ def test_score_kernel_timeline(name):
         if path:
             with open(path, "a") as f:
                 f.write(json.dumps(r) + "\n")
+
+
+def test_device_plan_matches_host_plan():
+    """wino_score_plan on this GPU equals the host-side split for its SM count and resident pairs (all 76
+    pairs are used at these shapes, so the device's pair count is what the plan shows)."""
+    import paper_2605_16941_gb300 as wino
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    for N, V in ((256, 126464), (2048, 134400), (1024, 126464)):
+        dev = wino.wino_score_plan(N, 4096, V)
+        pairs = dev["ctas"] // 2
+        host = wino.wino_score_plan_host(N, 4096, V, sms, pairs)
+        assert {k: host[k] for k in dev} == dev, (dev, host)
