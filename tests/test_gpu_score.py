@@ -18,6 +18,11 @@ SHAPES = [
     (384, 520, 777),
     (100, 64, 19400),   # last pair: one 256-wide tile with 200 valid columns
     (256, 128, 50000),  # several 256-wide tiles per pair and a 128-wide tail tile
+    # two-tile passes (two or more 256-row blocks):
+    (512, 64, 40000),   # one K slice: the second accumulator's MMAs deferred over a one-stage window
+    (520, 8, 300),      # d = 8 (K slice mostly zero fill), ragged last row block
+    (2048, 64, 129),    # a vocabulary narrower than one tile: every pass holds a single tile
+    (1024, 192, 70000),  # many passes per pair, odd tile counts (a single-tile last pass), ragged vocabulary
 ]
 
 
