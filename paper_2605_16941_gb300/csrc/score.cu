@@ -188,6 +188,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const bool leader = rank == 0;
     const int pair = blockIdx.x >> 1;
     uint64_t *const tl = a.timeline ? a.timeline + (size_t)blockIdx.x * kTimelineWords : nullptr;
+    // The record of an epilogue thread's last row block is stored after this CTA's arrival on the closing
+    // cluster barrier, so that the barrier's release does not wait for it.
+    float4 pend = make_float4(0.f, 0.f, 0.f, 0.f);
+    float pend_u = 0.f;
+    int64_t pend_idx = -1;
     if (tl && threadIdx.x == 0)
         tl[0] = ptx::globaltimer_ns();
 
@@ -455,9 +460,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 }
             }
             if (!aborted && row < a.N) {
-                a.part[row * a.G + col] = make_float4(r.m, (r.s0 + r.s1) + (r.s2 + r.s3), __int_as_float(r.am), r.tlog);
-                if (kEntropy)
-                    a.part_u[row * a.G + col] = (r.u0 + r.u1) + (r.u2 + r.u3);
+                if (pend_idx >= 0) {
+                    a.part[pend_idx] = pend;
+                    if (kEntropy)
+                        a.part_u[pend_idx] = pend_u;
+                }
+                pend = make_float4(r.m, (r.s0 + r.s1) + (r.s2 + r.s3), __int_as_float(r.am), r.tlog);
+                pend_u = (r.u0 + r.u1) + (r.u2 + r.u3);
+                pend_idx = row * a.G + col;
             }
         }
         if (tl && !leader && warp == 2 && lane == 0)
@@ -469,6 +479,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     __syncthreads();
     if (tl && threadIdx.x == 0)
         tl[5] = ptx::globaltimer_ns();
+    ptx::cluster_arrive_release();
+    if (pend_idx >= 0) {
+        a.part[pend_idx] = pend;
+        if (kEntropy)
+            a.part_u[pend_idx] = pend_u;
+    }
     if (threadIdx.x == 64) {
         // Warp 2 has passed griddepcontrol.wait, so the previous call's finish kernel, which clears the
         // status word, has completed: a failure recorded now belongs to this call.
@@ -477,7 +493,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         else if (*reinterpret_cast<volatile int32_t *>(&bars->abort))
             atomicExch(&a.status->current, (int32_t)WINO_ERR_DEVICE_TIMEOUT);
     }
-    ptx::cluster_sync();
+    ptx::cluster_wait_acquire();
     ptx::tc_fence_after();
     if (warp == 1)
         ptx::tmem_dealloc_pair(tmem, kTmemCols);

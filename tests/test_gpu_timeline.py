@@ -91,7 +91,7 @@ def _summaries(w, plan, T):
     return out
 
 
-@pytest.mark.parametrize("name", ["llada_b1", "llada_b8"])
+@pytest.mark.parametrize("name", ["tiny", "llada_b1", "llada_b8"])
 def test_score_kernel_timeline(name):
     w, plan, T = _run(name)
     path = os.environ.get("WINO_TIMELINE_RECORD")
