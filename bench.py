@@ -59,6 +59,16 @@ def load_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
+W_LAYOUTS = {"panels": "the LM head as 64-column panels (wino_lm_head_panels, made once before timing; "
+                      "WINO_OPT_W_PANELS)",
+             "rows": "the LM head row-major [V, d]"}
+
+
+def lm_head(wino, Wd, layout: str):
+    """The W argument of the steps for the chosen layout (the panel copy is made here, outside any timing)."""
+    return wino.wino_lm_head_panels(Wd) if layout == "panels" else Wd
+
+
 def config_dict(w):
     return {"workload": w.name, "N": w.N, "d": w.d, "V": w.V, "n_seq": w.n_seq, "blk_len": w.blk_len,
             "tau1": w.tau1, "tau2": w.tau2, "seed": w.seed,
@@ -234,14 +244,15 @@ def measure_configs(names, args, wino, ws, dev, sid, peaks, to_dev):
         if key not in w_cache:
             w_cache.clear()  # one extra LM head resident at a time
             W = ws.weights(w)
-            w_cache[key] = (W, to_dev(W))
+            w_cache[key] = (W, lm_head(wino, to_dev(W), args.w_layout))
         W, Wd = w_cache[key]
         st = ws.initial_state(w)
         Hd = [to_dev(ws.hidden_states(w, W, st, step=k)) for k in range(2)]
         tok = to_dev(st.tokens)
         counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device=dev)
         wsp = wino.workspace(w.N, w.d, w.V, device=dev)
-        p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len)
+        p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len,
+                             w_panels=args.w_layout == "panels")
 
         def step(i):
             wino.wino_step(Hd[i % 2], Wd, tok, p, counts, wsp, stream=sid)
@@ -258,7 +269,8 @@ def measure_configs(names, args, wino, ws, dev, sid, peaks, to_dev):
                      "ms_per_step": ms / args.steps, "rows_per_s": w.N / step_s,
                      "tflops_per_step": flops / step_s / 1e12,
                      "step_roofline_frac": max(t_flop, w_bytes / (peaks["hbm_gbs"] * 1e9)) / step_s,
-                     "kernel_roofline": kernel_roofline(w, w.N, peaks, score_avg_s)}
+                     "kernel_roofline": kernel_roofline(w, w.N, peaks, score_avg_s),
+                     "w_layout": W_LAYOUTS[args.w_layout]}
         del Hd, tok, wsp
     return out
 
@@ -431,13 +443,16 @@ def run_wino(args, rank, world, local_rank):
         a = np.ascontiguousarray(a)
         return torch.from_numpy(a.view(np.int16) if a.dtype == np.uint16 else a).to(dev)
 
-    Wd = to_dev(W)
+    W_rows = to_dev(W)  # row-major: wino_score_rows reads this layout
+    layout = "rows" if score_only else args.w_layout
+    Wd = lm_head(wino, W_rows, layout)
     Hd = [to_dev(h) for h in Hs]
     tok = to_dev(st.tokens)
     counts = torch.zeros((w.n_seq, 3), dtype=torch.int32, device=dev)
     wsp = wino.workspace(w.N, w.d, w.V, device=dev)
     p = wino.make_params(w.tau1, w.tau2, w.mask_id, w.n_seq, w.seq_len, st.blk_start, w.blk_len,
-                         compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m)
+                         compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m,
+                         w_panels=layout == "panels")
     if args.compact:  # row compaction needs room for the gathered rows
         wsp = wino.step_workspace(p, w.d, w.V, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -449,7 +464,7 @@ def run_wino(args, rank, world, local_rank):
 
     def step(i):
         if score_only:  # wino_score_rows alone (statistics of every row, optionally with H(p))
-            wino.wino_score_rows(Hd[i % n_h], Wd, None, am, pm, pt, wsp, stream=sid, entropy=ent)
+            wino.wino_score_rows(Hd[i % n_h], W_rows, None, am, pm, pt, wsp, stream=sid, entropy=ent)
         else:
             wino.wino_step(Hd[i % n_h], Wd, tok, p, counts, wsp, stream=sid)
 
@@ -466,7 +481,7 @@ def run_wino(args, rank, world, local_rank):
         with torch.cuda.graph(graph):
             for i in range(args.graph):
                 if score_only:
-                    wino.wino_score_rows(Hd[i % n_h], Wd, None, am, pm, pt, wsp, entropy=ent)
+                    wino.wino_score_rows(Hd[i % n_h], W_rows, None, am, pm, pt, wsp, entropy=ent)
                 else:
                     wino.wino_step(Hd[i % n_h], Wd, tok, p, counts, wsp)
         torch.cuda.synchronize(dev)
@@ -616,7 +631,7 @@ def run_wino(args, rank, world, local_rank):
             ws1 = wino.workspace(w.N, w.d, w.V, device=dev)
             wino.wino_step(Hd[0], Wd, tok1, p, cnt1, ws1, stream=sid)
             t_rows = to_dev(oracle.row_targets(st.tokens, st.blk_start, w.blk_len, w.mask_id))
-            wino.wino_score_rows(Hd[0], Wd, t_rows, am, pm, pt, ws1, stream=sid)
+            wino.wino_score_rows(Hd[0], W_rows, t_rows, am, pm, pt, ws1, stream=sid)
             torch.cuda.synchronize(dev)
             if wino.wino_read_device_status(ws1, stream=sid) != wino.WINO_OK:
                 raise RuntimeError("device status not OK in the parity step")
@@ -657,6 +672,7 @@ def run_wino(args, rank, world, local_rank):
             "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * te / e2e_steps},
         "gpu_launches": (3 if args.compact and not score_only else 2) * args.steps,  # (gather +) score + finish
         "clocks": clock_info,
+        "w_layout": W_LAYOUTS[layout],
         "cpu_baseline": cpu,
         "parity": parity,
         "configs": configs,
@@ -695,7 +711,7 @@ def run_loop(args):
         a = np.ascontiguousarray(a)
         return torch.from_numpy(a.view(np.int16) if a.dtype == np.uint16 else a).to(dev)
 
-    Wd = to_dev(W)
+    Wd = lm_head(wino, to_dev(W), args.w_layout)
     cache = {}
 
     def hidden(k, b0):
@@ -711,7 +727,7 @@ def run_loop(args):
         stats = driver(Wd, tok, prompt_len=w.prompt_len, blk_len=w.blk_len, n_blocks=w.n_blocks,
                        tau1=w.tau1, tau2=w.tau2, mask_id=w.mask_id, hidden=hidden, max_steps=4096,
                        compact=args.compact, no_shadow=args.no_shadow, draft_m=args.draft_m,
-                       skip_finished=args.skip_finished)
+                       skip_finished=args.skip_finished, w_panels=args.w_layout == "panels")
         return stats, tok
 
     t_gen = time.time()
@@ -733,7 +749,7 @@ def run_loop(args):
         "metric": METRIC, "mode": "decode_loop", "value": rows / t, "unit": UNIT, "n_gpus": 1,
         "steps": stats.total_steps, "ms_per_step": 1e3 * t / stats.total_steps, "seconds": t,
         "higher_is_better": True, "dtype": "bf16", "data": "synthetic", "config": config_dict(w),
-        "loop": {"reading": "bias U[0, 4 + 0.5 k] with k the global step index; a sequence whose block has no "
+        "w_layout": W_LAYOUTS[args.w_layout], "loop": {"reading": "bias U[0, 4 + 0.5 k] with k the global step index; a sequence whose block has no "
                             "MASK is frozen until the batch's block is done",
                  "steps_per_block": [b.steps for b in stats.blocks],
                  "drafted_per_block": [b.drafted for b in stats.blocks],
@@ -785,6 +801,8 @@ def main():
                     help="with --loop: score only the sequences whose block still has a MASK")
     ap.add_argument("--python-loop", action="store_true",
                     help="with --loop: step from the Python driver (loop.decode) instead of the library's loop")
+    ap.add_argument("--w-layout", choices=sorted(W_LAYOUTS), default="panels",
+                    help="LM head layout the steps read (wino_score_rows always reads row-major W)")
     ap.add_argument("--cpu-budget-s", type=float, default=15.0)
     ap.add_argument("--ref-budget-s", type=float, default=90.0)
     args = ap.parse_args()

@@ -132,6 +132,15 @@ typedef struct {
 #define WINO_OPT_COMPACT 4
 
 /*
+ * WINO_OPT_W_PANELS (wino_step, wino_step_static_scratch, wino_decode): the
+ * W argument is the panel copy of the LM head written by
+ * wino_lm_head_panels(), not the row-major [V, d] matrix (d then a multiple
+ * of 64 and (d/64)*V at most 2^30, else WINO_ERR_SHAPE).  The results are
+ * bit-identical to those with row-major W.
+ */
+#define WINO_OPT_W_PANELS 8
+
+/*
  * Bytes of scratch wino_score_rows needs for N rows of dimension d over a
  * vocabulary of V entries, with or without the entropy output: status words,
  * per-sequence tickets, per-row partial softmax records (R = min(ceil(V/128),
@@ -156,6 +165,26 @@ WINO_API int wino_workspace_size(int64_t N, int64_t d, int64_t V, size_t *bytes)
  * for wino_workspace_size.
  */
 WINO_API int wino_workspace_size_step(const wino_params *p, int64_t d, int64_t V, size_t *bytes);
+
+/*
+ * The LM head re-laid out in d/64 panels of 64 columns (a weight layout of
+ * this library; the paper has no counterpart):
+ *     Wp[k][v][c] = W[v][64k + c],  k < d/64, v < V, c < 64,
+ * bf16, V*d*2 bytes (the size of W).  A step with WINO_OPT_W_PANELS reads W
+ * through this copy: every copy of the score kernel (bn/2 vocabulary rows x
+ * one 64-wide K slice, 15-16 KB) is then one contiguous block of HBM instead
+ * of bn/2 pieces of 128 bytes, 2*d bytes apart, and the W stream runs closer
+ * to the HBM peak (about 2 % faster steps at one 256-row block, 1 % at
+ * N = 2048).  Make the copy once per LM head and keep it while W does not
+ * change; the library does not track W.
+ *   W   [V, d] bf16 (uint16_t bits), device, 16-byte aligned; not modified
+ *   Wp  device, 16-byte aligned, V*d*2 bytes, not overlapping W; written
+ *       asynchronously on `stream`
+ * d must be a multiple of 64 and (d/64)*V at most 2^30.  Returns WINO_ERR_ARG
+ * for null, misaligned or overlapping buffers, WINO_ERR_SHAPE for other sizes,
+ * WINO_ERR_CUDA if the launch fails.
+ */
+WINO_API int wino_lm_head_panels(const uint16_t *W, int64_t d, int64_t V, uint16_t *Wp, void *stream);
 
 /*
  * Fused LM-head GEMM + full-vocabulary softmax statistics (the p_theta(.|Y~)

@@ -30,11 +30,12 @@ FLAG_NONE, FLAG_DRAFT, FLAG_DRAFT_FALLBACK, FLAG_REMASK, FLAG_DRAFT_IS_MASK, FLA
 WINO_OPT_FREEZE_FINISHED = 1
 WINO_OPT_NO_SHADOW = 2
 WINO_OPT_COMPACT = 4
+WINO_OPT_W_PANELS = 8
 
 EXPORTS = ("wino_workspace_size", "wino_workspace_size_step", "wino_score_rows", "wino_draft_verify", "wino_step",
            "wino_step_static_scratch", "wino_read_device_status", "wino_profile_begin", "wino_profile_end",
            "wino_selftest_wait_timeout", "wino_status_string", "wino_version", "wino_decode", "wino_timeline_begin",
-           "wino_timeline_end", "wino_score_plan", "wino_score_plan_host")
+           "wino_timeline_end", "wino_score_plan", "wino_score_plan_host", "wino_lm_head_panels")
 
 # 64-bit words per CTA in a score-kernel timeline (wino_timeline_begin)
 TIMELINE_WORDS = 8
@@ -88,6 +89,8 @@ def lib() -> C.CDLL:
         L.wino_draft_verify.argtypes = [vp, vp, vp, vp, C.POINTER(WinoParams), vp, vp, vp]
         L.wino_step.restype = C.c_int
         L.wino_step.argtypes = [vp, vp, i64, i64, vp, C.POINTER(WinoParams), vp, vp, vp, sz, vp]
+        L.wino_lm_head_panels.restype = C.c_int
+        L.wino_lm_head_panels.argtypes = [vp, i64, i64, vp, vp]
         L.wino_step_static_scratch.restype = C.c_int
         L.wino_step_static_scratch.argtypes = [vp, vp, i64, i64, vp, C.POINTER(WinoParams), vp, vp, vp]
         L.wino_read_device_status.restype = C.c_int
@@ -175,11 +178,12 @@ def workspace(N: int, d: int, V: int, device=None):
 def make_params(tau1: float, tau2: float, mask_id: int, n_seq: int, seq_len: int, blk_start: int, blk_len: int,
                 max_steps: int = 4096, freeze_finished: bool = False, step_index: int = 0,
                 last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0,
-                active_seq=None, n_active: int | None = None) -> WinoParams:
+                active_seq=None, n_active: int | None = None, w_panels: bool = False) -> WinoParams:
     """wino_params; ``draft_m`` > 0 selects fixed-M drafting (naive parallel sampling, Sec. 3);
-    ``active_seq`` (device int32) lists the sequences a wino_step scores and updates (default: all)."""
+    ``active_seq`` (device int32) lists the sequences a wino_step scores and updates (default: all);
+    ``w_panels``: the W passed to the step is the panel copy of ``wino_lm_head_panels``."""
     opts = ((WINO_OPT_FREEZE_FINISHED if freeze_finished else 0) | (WINO_OPT_NO_SHADOW if no_shadow else 0) |
-            (WINO_OPT_COMPACT if compact else 0))
+            (WINO_OPT_COMPACT if compact else 0) | (WINO_OPT_W_PANELS if w_panels else 0))
     if active_seq is not None and n_active is None:
         n_active = int(active_seq.numel())
     return WinoParams(tau1, tau2, mask_id, n_seq, seq_len, blk_start, blk_len, max_steps, opts, step_index,
@@ -204,11 +208,27 @@ def wino_draft_verify(tokens, argmax, pmax, ptarget, params: WinoParams, counts,
                                    _ptr(counts), _ptr(flags), _stream(stream)), "wino_draft_verify")
 
 
+def _vocab(W, params: WinoParams) -> int:
+    """V from W's shape: [V, d] row-major, or [d/64, V, 64] for a panel copy (WINO_OPT_W_PANELS)."""
+    return int(W.shape[1] if params.options & WINO_OPT_W_PANELS else W.shape[0])
+
+
+def wino_lm_head_panels(W, Wp=None, stream=None):
+    """The panel copy Wp[k][v][c] = W[v][64k + c] of a [V, d] bf16 LM head, as a [d/64, V, 64] tensor (written
+    into ``Wp`` when given, else allocated by PyTorch); pass it as W with ``make_params(..., w_panels=True)``."""
+    import torch
+    V, d = int(W.shape[0]), int(W.shape[1])
+    if Wp is None:
+        Wp = torch.empty((d // 64, V, 64), dtype=W.dtype, device=W.device)
+    _check(lib().wino_lm_head_panels(_ptr(W), d, V, _ptr(Wp), _stream(stream)), "wino_lm_head_panels")
+    return Wp
+
+
 def wino_step(H, W, tokens, params: WinoParams, counts, ws, flags=None, stream=None, *, d: int | None = None,
               V: int | None = None) -> None:
     """One whole WINO step in place on ``tokens``."""
     d = int(H.shape[1]) if d is None else d
-    V = int(W.shape[0]) if V is None else V
+    V = _vocab(W, params) if V is None else V
     ws_bytes = ws.numel() * ws.element_size()
     _check(lib().wino_step(_ptr(H), _ptr(W), d, V, _ptr(tokens), C.byref(params), _ptr(counts), _ptr(flags),
                            _ptr(ws), ws_bytes, _stream(stream)), "wino_step")
@@ -218,7 +238,7 @@ def wino_step_static_scratch(H, W, tokens, params: WinoParams, counts, flags=Non
                              d: int | None = None, V: int | None = None) -> None:
     """wino_step with the library's fixed device scratch instead of a caller workspace (allocates nothing)."""
     d = int(H.shape[1]) if d is None else d
-    V = int(W.shape[0]) if V is None else V
+    V = _vocab(W, params) if V is None else V
     _check(lib().wino_step_static_scratch(_ptr(H), _ptr(W), d, V, _ptr(tokens), C.byref(params), _ptr(counts),
                                           _ptr(flags), _stream(stream)), "wino_step_static_scratch")
 
@@ -233,8 +253,11 @@ def wino_decode(W, tokens, params: WinoParams, n_blocks: int, hidden, counts, co
     MASK are stepped.  Returns (status, per-block (steps, drafted, re-masked, at-least-one drafts,
     sequences stepped summed over the steps), next step index); the status is
     WINO_OK or the error that stopped the loop (an exception raised by ``hidden`` is re-raised)."""
-    d = int(W.shape[1]) if d is None else d
-    V = int(W.shape[0]) if V is None else V
+    if params.options & WINO_OPT_W_PANELS:  # [d/64, V, 64]
+        d = int(W.shape[0]) * 64 if d is None else d
+    else:
+        d = int(W.shape[1]) if d is None else d
+    V = _vocab(W, params) if V is None else V
     held, failure = [None], []
 
     def cb(user, k, blk_start):

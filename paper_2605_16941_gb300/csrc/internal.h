@@ -116,6 +116,7 @@ struct ScoreArgs {
     int32_t *tickets;   // [n_tickets], cleared here for the finish kernel
     int32_t n_tickets;
     uint64_t *timeline;        // nullptr, or [gridDim.x][kTimelineWords] stamps of this launch
+    int32_t w_panels;          // W's tensor map is over the panel copy [d/64 * V, 64]: row v of K slice kb at kb * V + v
 };
 
 struct FinishArgs {
@@ -168,6 +169,9 @@ cudaError_t launch_gather_active(const uint16_t *H, uint16_t *Hc, int32_t *targe
                                  const wino_params &p, int64_t rows, int64_t d, cudaStream_t stream);
 cudaError_t launch_gather_compact(const uint16_t *H, uint16_t *Hc, const int32_t *tokens, const wino_params &p,
                                   int64_t d, cudaStream_t stream);
+
+// Wp[k][v][c] = W[v][64k + c] (wino_lm_head_panels); d a multiple of 64, (d/64) * V <= 2^30.
+cudaError_t launch_panels(const uint16_t *W, uint16_t *Wp, int64_t d, int64_t V, int sm_count, cudaStream_t stream);
 
 cudaError_t launch_draft_verify(int32_t *tokens, const int32_t *argmax, const float *pmax, const float *ptarget,
                                 const wino_params &p, int32_t *counts, int8_t *flags, cudaStream_t stream);

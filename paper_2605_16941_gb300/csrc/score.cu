@@ -264,9 +264,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer (both CTAs)
         const int half_bn = a.bn >> 1;  // W rows each CTA stages per tile
+        // W map coordinates of (K slice kb, vocabulary row v): (64 kb, v) in row-major W, (0, kb V + v) in the
+        // panel copy
+        auto w_x = [&](int kb) { return a.w_panels ? 0 : kb * kBK; };
+        auto w_y = [&](int kb, int v) { return a.w_panels ? kb * a.V + v : v; };
         if (lane == 0 && grp < a.n_mb)
             for (int kb = 0; kb < min(a.n_kb, kPrefetchSlices); ++kb)
-                ptx::tma_prefetch_2d(&tmW, kb * kBK, col * a.bn + (int)rank * half_bn);
+                ptx::tma_prefetch_2d(&tmW, w_x(kb), w_y(kb, col * a.bn + (int)rank * half_bn));
         ptx::grid_dep_wait();
         const uint64_t pol_h = ptx::policy_evict_last();    // H is re-read for every item
         const uint64_t pol_w = ptx::policy_evict_normal();  // W is shared by the row-block groups
@@ -295,11 +299,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         if (leader)
                             ptx::mbar_arrive_expect_tx(full(stage), stage_tx);
                         ptx::tma_load_2d_pair(sA(stage), &tmH, bar, kb * kBK, mb * kPairM + (int)rank * kBM, pol_h);
-                        ptx::tma_load_2d_pair(sB(stage, 0), &tmW, bar, kb * kBK, vt * a.bn + (int)rank * half_bn,
-                                              pol_w);
+                        ptx::tma_load_2d_pair(sB(stage, 0), &tmW, bar, w_x(kb),
+                                              w_y(kb, vt * a.bn + (int)rank * half_bn), pol_w);
                         if (two)
-                            ptx::tma_load_2d_pair(sB(stage, 1), &tmW, bar, kb * kBK,
-                                                  (vt + a.G) * a.bn + (int)rank * half_bn, pol_w);
+                            ptx::tma_load_2d_pair(sB(stage, 1), &tmW, bar, w_x(kb),
+                                                  w_y(kb, (vt + a.G) * a.bn + (int)rank * half_bn), pol_w);
                         if (tl && first)
                             tl[2] = ptx::globaltimer_ns();
                         first = false;

@@ -20,6 +20,7 @@ namespace {
 constexpr int64_t kMaxN = int64_t(1) << 24;
 constexpr int64_t kMaxD = 65536;
 constexpr int64_t kMaxV = int64_t(1) << 27;
+constexpr int64_t kMaxPanelRows = int64_t(1) << 30;  // (d/64) * V of a panel copy: its row coordinates stay in int32
 constexpr size_t kAlign = 256;
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -215,9 +216,11 @@ int check_params(const wino_params *p)
 
 // Score N rows into (argmax, pmax, ptarget), and with `step` also apply Eq. 4:
 // the score kernel followed by the finish kernel.
-int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, int64_t V, const TargetSource &ts,
-                     int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws, size_t ws_bytes,
-                     const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags, cudaStream_t stream)
+// W is row-major [V, d], or with w_panels the panel copy [d/64][V][64] of wino_lm_head_panels.
+int score_and_finish(const uint16_t *H, const uint16_t *W, bool w_panels, int64_t N, int64_t d, int64_t V,
+                     const TargetSource &ts, int32_t *argmax, float *pmax, float *ptarget, float *entropy, void *ws,
+                     size_t ws_bytes, const wino_params *step, int32_t *tokens, int32_t *counts, int8_t *flags,
+                     cudaStream_t stream)
 {
     DeviceInfo info;
     int rc = device_info(&info);
@@ -235,7 +238,9 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     CUtensorMap tmH, tmW;
     if ((rc = tensor_map(H, N, d, kBM, &tmH)) != WINO_OK)
         return rc;
-    if ((rc = tensor_map(W, V, d, sch.bn / 2, &tmW)) != WINO_OK)
+    // one 16-byte-aligned map row per (K slice, vocabulary row) of the panel copy
+    if ((rc = w_panels ? tensor_map(W, d / kBK * V, kBK, sch.bn / 2, &tmW) : tensor_map(W, V, d, sch.bn / 2, &tmW)) !=
+        WINO_OK)
         return rc;
     uint8_t *w8 = static_cast<uint8_t *>(ws);
     ScoreArgs a{};
@@ -258,6 +263,7 @@ int score_and_finish(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d,
     a.tickets = reinterpret_cast<int32_t *>(w8 + L.tickets);
     a.n_tickets = step ? step->n_seq : 0;
     a.timeline = timeline_slot((unsigned)(2 * a.n_groups * a.G));
+    a.w_panels = w_panels ? 1 : 0;
     prof_record(0, stream);
     if (launch_score(tmH, tmW, a, entropy != nullptr, stream) != cudaSuccess)
         return WINO_ERR_CUDA;
@@ -364,7 +370,7 @@ int wino_score_rows(const uint16_t *H, const uint16_t *W, int64_t N, int64_t d, 
         return WINO_ERR_SHAPE;
     TargetSource ts{};
     ts.target = target;
-    return score_and_finish(H, W, N, d, V, ts, argmax, pmax, ptarget, entropy, ws, ws_bytes, nullptr, nullptr,
+    return score_and_finish(H, W, false, N, d, V, ts, argmax, pmax, ptarget, entropy, ws, ws_bytes, nullptr, nullptr,
                             nullptr, nullptr, static_cast<cudaStream_t>(stream));
 }
 
@@ -408,6 +414,9 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
     const int64_t N = step_rows(*p);  // rows scored
     if (!shape_ok(N, d, V) || p->mask_id >= V)
         return WINO_ERR_SHAPE;
+    const bool w_panels = (p->options & WINO_OPT_W_PANELS) != 0;
+    if (w_panels && (d % kBK != 0 || d / kBK * V > kMaxPanelRows))
+        return WINO_ERR_SHAPE;
     const WsLayout L = ws_layout(N, V);
     if (ws_bytes < step_ws_bytes(*p, d, V))
         return WINO_ERR_WORKSPACE;
@@ -434,7 +443,8 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
             return WINO_ERR_CUDA;
         TargetSource tsa{};
         tsa.target = tgt;
-        return score_and_finish(Hc, W, N, d, V, tsa, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s);
+        return score_and_finish(Hc, W, w_panels, N, d, V, tsa, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts,
+                                flags, s);
     }
     if (compact) {  // gather the one row per position Eq. 4 reads, behind the workspace proper
         DeviceInfo info;
@@ -445,7 +455,28 @@ int wino_step(const uint16_t *H, const uint16_t *W, int64_t d, int64_t V, int32_
             return WINO_ERR_CUDA;
         Hs = Hc;
     }
-    return score_and_finish(Hs, W, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags, s);
+    return score_and_finish(Hs, W, w_panels, N, d, V, ts, am, pm, pt, nullptr, ws, ws_bytes, p, tokens, counts, flags,
+                            s);
+}
+
+int wino_lm_head_panels(const uint16_t *W, int64_t d, int64_t V, uint16_t *Wp, void *stream)
+{
+    const Range range("wino_lm_head_panels");
+    if (!W || !Wp || !aligned(W, 16) || !aligned(Wp, 16))
+        return WINO_ERR_ARG;
+    if (d < kBK || d > kMaxD || d % kBK != 0 || V < 2 || V > kMaxV || d / kBK * V > kMaxPanelRows)
+        return WINO_ERR_SHAPE;
+    const uintptr_t bytes = (uintptr_t)V * (uintptr_t)d * 2u;
+    const uintptr_t w0 = reinterpret_cast<uintptr_t>(W), p0 = reinterpret_cast<uintptr_t>(Wp);
+    if (w0 < p0 + bytes && p0 < w0 + bytes)
+        return WINO_ERR_ARG;  // the copy cannot be made in place
+    DeviceInfo info;
+    int rc = device_info(&info);
+    if (rc != WINO_OK)
+        return rc;
+    if (launch_panels(W, Wp, d, V, info.sm_count, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return WINO_ERR_CUDA;
+    return WINO_OK;
 }
 
 int wino_profile_begin(int max_launches)

@@ -49,11 +49,18 @@ def resume_point(k: int, blk_start: int, counts, *, prompt_len: int, blk_len: in
     return (b + 1 if done else b), k + 1
 
 
+def _head_dims(W, w_panels: bool) -> tuple[int, int]:
+    """(d, V) of an LM head given row-major [V, d] or as a panel copy [d/64, V, 64]."""
+    if w_panels:
+        return int(W.shape[0]) * 64, int(W.shape[1])
+    return int(W.shape[1]), int(W.shape[0])
+
+
 def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float, mask_id: int,
            hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
            on_step: Callable | None = None, last_change=None, no_shadow: bool = False,
            compact: bool = False, draft_m: int = 0, trajectory: list | None = None, start_block: int = 0,
-           start_step: int = 0, skip_finished: bool = False) -> LoopStats:
+           start_step: int = 0, skip_finished: bool = False, w_panels: bool = False) -> LoopStats:
     """Decode ``n_blocks`` blocks of ``tokens`` (int32 [n_seq, S], device) in place.
 
     ``hidden(k, blk_start)`` returns the device bf16 hidden states [2*n_seq*blk_len, d]
@@ -75,19 +82,21 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     ``skip_finished``: each step scores only the sequences whose block still has a MASK (an
     active-sequence list, ``wino_params.active_seq``); the states are those of the frozen
     sequences without it, and ``on_step`` sees zero counts for the sequences left out.
+    ``w_panels``: ``W`` is the panel copy of ``wino_lm_head_panels`` ([d/64, V, 64]), same results.
     """
     import numpy as np
     import torch
 
     n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
-    d, V = int(W.shape[1]), int(W.shape[0])
+    d, V = _head_dims(W, w_panels)
     rows_per_seq = (1 if (no_shadow or compact) else 2) * blk_len  # rows scored per sequence and step
     dev = tokens.device
     ts = stream if stream is not None else torch.cuda.current_stream(dev)  # every copy goes on the step's stream
     active_d = torch.arange(n_seq, dtype=torch.int32, device=dev) if skip_finished else None
     active_h = torch.zeros(n_seq, dtype=torch.int32, pin_memory=True) if skip_finished else None
     p0 = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact,
-                     draft_m=draft_m, active_seq=active_d, n_active=n_seq if skip_finished else None)
+                     draft_m=draft_m, active_seq=active_d, n_active=n_seq if skip_finished else None,
+                     w_panels=w_panels)
     ws = torch.zeros(wino_workspace_size_step(p0, d, V), dtype=torch.uint8, device=dev)
     counts = torch.zeros((n_seq, 3), dtype=torch.int32, device=dev)
     flags = torch.zeros((n_seq, blk_len), dtype=torch.int8, device=dev)
@@ -104,7 +113,8 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
     for b in range(start_block, n_blocks):
         b0 = prompt_len + b * blk_len
         p = make_params(tau1, tau2, mask_id, n_seq, S, b0, blk_len, max_steps, freeze_finished=True,
-                        last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
+                        last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m,
+                        w_panels=w_panels)
         bs = BlockStats(block=b, blk_start=b0)
         active = list(range(n_seq))  # a new block: every sequence takes part
         while True:
@@ -156,20 +166,22 @@ def decode(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: flo
 def decode_native(W, tokens, *, prompt_len: int, blk_len: int, n_blocks: int, tau1: float, tau2: float,
                   mask_id: int, hidden: Callable[[int, int], object], max_steps: int = 4096, stream=None,
                   last_change=None, no_shadow: bool = False, compact: bool = False, draft_m: int = 0,
-                  start_block: int = 0, start_step: int = 0, skip_finished: bool = False) -> LoopStats:
+                  start_block: int = 0, start_step: int = 0, skip_finished: bool = False,
+                  w_panels: bool = False) -> LoopStats:
     """``decode`` with the step loop run by the library (``wino_decode``): the same steps, states and
     statistics, with one callback into Python per step (for the hidden states) instead of the whole
     per-step bookkeeping.  No ``on_step`` or ``trajectory``; errors raise ``WinoError``.
-    ``skip_finished`` as in ``decode``: the library keeps the active-sequence list."""
+    ``skip_finished`` as in ``decode``: the library keeps the active-sequence list; ``w_panels`` as in ``decode``."""
     import torch
 
     n_seq, S = int(tokens.shape[0]), int(tokens.shape[1])
-    d, V = int(W.shape[1]), int(W.shape[0])
+    d, V = _head_dims(W, w_panels)
     rows_per_seq = (1 if (no_shadow or compact) else 2) * blk_len
     dev = tokens.device
     ts = stream if stream is not None else torch.cuda.current_stream(dev)
     p = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, max_steps, freeze_finished=True,
-                    last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m)
+                    last_change=last_change, no_shadow=no_shadow, compact=compact, draft_m=draft_m,
+                    w_panels=w_panels)
     active_buf = torch.zeros(n_seq, dtype=torch.int32, device=dev) if skip_finished else None
     p_ws = make_params(tau1, tau2, mask_id, n_seq, S, prompt_len, blk_len, no_shadow=no_shadow, compact=compact,
                        active_seq=active_buf, n_active=n_seq if skip_finished else None)  # sized for every list
