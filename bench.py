@@ -140,9 +140,9 @@ class ClockSampler:
                 "samples": len(sm), "samples_in_timed_region": len(inside)}
 
 
-def ncu_traffic(workload_name: str):
-    """DRAM bytes per score launch from the committed ncu capture, if it was taken on this workload and
-    none of the score kernel's source files has changed since (else None)."""
+def ncu_traffic(workload_name: str, layout: str = "panels"):
+    """DRAM bytes per score launch from the committed ncu capture, if it was taken on this workload with this
+    LM-head layout and none of the score kernel's source files has changed since (else None)."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "score_kernel_traffic.txt")) as f:
@@ -153,7 +153,8 @@ def ncu_traffic(workload_name: str):
                 h.update(f.read())
     except (OSError, ValueError, KeyError, TypeError):
         return None
-    if rec.get("workload") != workload_name or rec.get("sources_sha256_prefix") != h.hexdigest()[:16]:
+    if rec.get("workload") != workload_name or rec.get("sources_sha256_prefix") != h.hexdigest()[:16] or \
+            rec.get("w_layout", "rows") != layout:
         return None
     return float(rec["dram_bytes_read"]) + float(rec["dram_bytes_write"])
 
@@ -661,7 +662,7 @@ def run_wino(args, rank, world, local_rank):
         "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": cfg,
         "roofline": {**{k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac")},
-                     "traffic": ncu_traffic(w.name), "kernel": "score_kernel (fused LM-head GEMM + online vocab softmax)",
+                     "traffic": ncu_traffic(w.name, layout), "kernel": "score_kernel (fused LM-head GEMM + online vocab softmax)",
                      **{k: v for k, v in roof.items() if k not in ("bound", "achieved", "peak", "unit", "frac")},
                      "launches_timed": score_n, "peak_source": peak_src,
                      "timing": "per-launch CUDA events around the score kernel over a second region of K steps"},

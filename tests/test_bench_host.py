@@ -29,7 +29,8 @@ def _sha(csrc, names):
 
 
 def test_ncu_traffic_is_tied_to_the_kernel_sources(tmp_path, monkeypatch):
-    """A traffic record counts only while every source file the score kernel is built from is unchanged."""
+    """A traffic record counts only for its workload and LM-head layout, and only while every source file the score
+    kernel is built from is unchanged."""
     rec = json.loads((ROOT / "profiles" / "score_kernel_traffic.txt").read_text())
     want = float(rec["dram_bytes_read"]) + float(rec["dram_bytes_write"])
     fresh = rec["sources_sha256_prefix"] == _sha(ROOT / "paper_2605_16941_gb300" / "csrc", rec["score_kernel_sources"])
@@ -40,6 +41,8 @@ def test_ncu_traffic_is_tied_to_the_kernel_sources(tmp_path, monkeypatch):
     (tmp_path / "profiles" / "score_kernel_traffic.txt").write_text(json.dumps(rec))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     assert bench.ncu_traffic(rec["workload"]) == want
+    other = "rows" if rec.get("w_layout", "rows") == "panels" else "panels"
+    assert bench.ncu_traffic(rec["workload"], other) is None  # taken with the other LM-head layout
     for name in rec["score_kernel_sources"]:  # a change to any source the kernel is built from voids it
         f = csrc / name
         old = f.read_bytes()
