@@ -235,7 +235,8 @@ WINO_API int wino_draft_verify(int32_t *tokens, const int32_t *argmax, const flo
  * for block rows), every row is scored as in wino_score_rows, and Eq. 4 is
  * applied as in wino_draft_verify.
  *   H [2*n_seq*blk_len, d] bf16 rows in [s][kind][l] order (with
- *     WINO_OPT_NO_SHADOW: [n_seq*blk_len, d], block rows only); W [V, d] bf16.
+ *     WINO_OPT_NO_SHADOW: [n_seq*blk_len, d], block rows only); W [V, d] bf16,
+ *     or with WINO_OPT_W_PANELS its panel copy (wino_lm_head_panels).
  * If a device wait expired, tokens are left unchanged and every counts entry
  * is set to WINO_ERR_DEVICE_TIMEOUT.
  */
@@ -308,7 +309,8 @@ WINO_API int wino_step_static_scratch(const uint16_t *H, const uint16_t *W, int6
  *                are copied here and the at-least-one drafts counted
  *   next_step    host or NULL: the global index after the last step run;
  *                with the block that follows, the point to resume from
- * counts, flags (optional), ws and ws_bytes are as for wino_step.
+ * W (row-major, or the panel copy with WINO_OPT_W_PANELS), counts, flags
+ * (optional), ws and ws_bytes are as for wino_step.
  */
 typedef const uint16_t *(*wino_hidden_fn)(void *user, int32_t step, int32_t blk_start);
 typedef struct {
