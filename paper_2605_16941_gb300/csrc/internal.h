@@ -21,9 +21,11 @@ namespace wino {
 //   single tiles: the accumulators alternate, so the epilogue of one tile
 //     overlaps the MMAs of the next; stages of 16 KB + bn*64 B, up to 7 of them
 //     (the most bytes in flight, for shapes bound by the W stream from HBM);
-//   two-tile passes: a stage holds one H slice and the slices of two tiles,
-//     multiplied into both accumulators, so H is staged once per two tiles
-//     (a quarter fewer bytes delivered per SM and MMA, for tensor-bound shapes).
+//   passes (tensor-bound shapes): a stage holds three slots multiplied into
+//     both accumulators, a quarter fewer bytes delivered per SM and MMA.  Two
+//     row blocks of a group share each W slice (row-pair sweep: H, W, H), so
+//     the group reads W from HBM once per two blocks; a block without a partner
+//     shares its H slice between two tiles (tile-pair sweep: H, W, W).
 constexpr int kPairM = 256;  // rows per pair tile (UMMA M)
 constexpr int kBM = 128;     // rows per CTA
 constexpr int kBN = 256;     // largest tile width (UMMA N); TMEM column stride of the two accumulators
@@ -75,9 +77,9 @@ __device__ __forceinline__ int32_t row_target(const TargetSource &ts, int64_t ro
 
 // Work split of the score kernel.  The 256-row blocks are spread over n_groups
 // groups of G CTA pairs; pair c serves row blocks c % n_groups (+ n_groups, ...)
-// and, within each, vocabulary tiles c / n_groups (+ G, ...), two per pass.  The G pairs of a
+// and, within each, vocabulary tiles c / n_groups (+ G, ...).  The G pairs of a
 // group walk the vocabulary side by side, so all groups read the same W tiles
-// at the same time (W streams from HBM about once), and each CTA keeps its
+// at the same time (W streams from HBM once per sweep), and each CTA keeps its
 // running softmax state per row across its tiles and writes ONE partial record
 // per (row, pair of the group): G records per row.
 constexpr int kMaxRecordsPerRow = 256;
@@ -105,9 +107,9 @@ struct ScoreArgs {
     int32_t N, d, V;
     int32_t n_mb, n_vt, n_kb;  // n_mb: 256-row blocks, n_vt: vocabulary tiles of bn columns
     int32_t bn;                // tile width (multiple of 16, kMinBN..kBN)
-    int32_t two;               // 1: two-tile passes, 0: single tiles (see above)
+    int32_t two;               // 1: passes, 0: single tiles (see above)
     int32_t stages;            // ring stages, 2..kMaxStages
-    uint32_t stage_bytes;      // 16 KB + (1 + two) * stage_bytes_w(bn)
+    uint32_t stage_bytes;      // 16 KB + stage_bytes_w(bn) + a pass's third slot (W, or 16 KB of H)
     int32_t n_groups, G;
     TargetSource ts;
     float4 *part;       // [N][G]

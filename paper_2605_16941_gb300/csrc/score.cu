@@ -17,18 +17,24 @@
 //     block): the two accumulators alternate between consecutive tiles, so
 //     the epilogue of one tile overlaps the MMAs of the next, and the ring has
 //     up to 7 stages, the most W bytes in flight per SM;
-//   two-tile passes, for tensor-bound shapes: every K slice of H is staged
-//     once and multiplied with the slices of two tiles into both accumulators,
-//     a quarter fewer bytes delivered per SM and MMA.  The accumulators then
-//     fill TMEM, so a pass's MMAs into the first accumulator start as soon as
-//     the epilogue has read it, and its MMAs into the second accumulator for
-//     the first ring stages are deferred until the epilogue has read that one
-//     too (the stages are released after those).
+//   passes, for tensor-bound shapes: a stage holds three 16 KB slots and
+//     feeds both accumulators, a quarter fewer bytes delivered per SM and MMA
+//     than single tiles.  A group of pairs that owns two or more row blocks
+//     takes them two at a time (row-pair sweeps): the two blocks' H slices
+//     and one tile's W slice, so every W slice staged serves both blocks and
+//     the group streams W from HBM once per two blocks.  A block left without
+//     a partner is swept alone (tile-pair sweeps): its H slice and the slices
+//     of two tiles.  The accumulators then fill TMEM, so a pass's MMAs into
+//     the first accumulator start as soon as the epilogue has read it, and
+//     its MMAs into the second accumulator for the first ring stages are
+//     deferred until the epilogue has read that one too (the stages are
+//     released after those).
 //
 // Kernel structure (persistent, clusters of 2 CTAs = one SM pair, 192 threads each):
-//   warp 0  TMA producer (both CTAs): per K slice, its 128 rows of H and its
-//           bn/2 of the (one or two) tiles' W rows into the ring; both CTAs'
-//           copies complete on the LEADER's stage barrier;
+//   warp 0  TMA producer (both CTAs): per K slice, its 128 rows of H (of one
+//           or two row blocks) and its bn/2 of the (one or two) tiles' W rows
+//           into the ring; both CTAs' copies complete on the LEADER's stage
+//           barrier;
 //   warp 1  TMEM allocation (both CTAs, all 512 columns) and, in the leader
 //           only, the MMA issuer: 4 x (M256 Nbn K16) per stage and tile,
 //           committing stage release and accumulator-ready to both CTAs
@@ -173,7 +179,7 @@ __device__ __forceinline__ void fold_tile(RowState &r, uint32_t tbase, int v0, i
     }
 }
 
-// kTwo: two-tile passes (ScoreArgs::two == 1), else single tiles.
+// kTwo: passes (ScoreArgs::two == 1: row-pair and tile-pair sweeps), else single tiles.
 template <bool kEntropy, bool kTwo>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW,
@@ -188,11 +194,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const bool leader = rank == 0;
     const int pair = blockIdx.x >> 1;
     uint64_t *const tl = a.timeline ? a.timeline + (size_t)blockIdx.x * kTimelineWords : nullptr;
-    // The record of an epilogue thread's last row block is stored after this CTA's arrival on the closing
-    // cluster barrier, so that the barrier's release does not wait for it.
-    float4 pend = make_float4(0.f, 0.f, 0.f, 0.f);
-    float pend_u = 0.f;
-    int64_t pend_idx = -1;
+    // The records of an epilogue thread's last sweep (one row, or two in a row-pair sweep) are stored after
+    // this CTA's arrival on the closing cluster barrier, so that the barrier's release does not wait for them.
+    float4 pend[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+    float pend_u[2] = {0.f, 0.f};
+    int64_t pend_idx[2] = {-1, -1};
     if (tl && threadIdx.x == 0)
         tl[0] = ptx::globaltimer_ns();
 
@@ -247,7 +253,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
     const int grp = pair % a.n_groups;  // 256-row blocks grp, grp + n_groups, ...
     const int col = pair / a.n_groups;  // vocabulary tiles col, col + G, ...
-    const int vstep = kTwo ? 2 * a.G : a.G;  // tiles per item: 1, or 2 (col + 2jG and col + (2j+1)G)
+    // Sweeps over the pair's vocabulary tiles.  Single tiles: one sweep per row block, one tile per item.
+    // Passes: row blocks mb and mb + n_groups together (row-pair sweep: item = one tile of both blocks, so
+    // each W slice staged serves both and the group reads W once per two blocks), or a block left without
+    // a partner alone (tile-pair sweep: item = tiles vt and vt + G of that block).
+    const int mb_step = kTwo ? 2 * a.n_groups : a.n_groups;
+    const int vstep = kTwo ? 2 * a.G : a.G;  // tiles per item of a single-tile or tile-pair sweep
 
     if (warp >= 2 || !tmem_ok) {
         ptx::grid_dep_wait();
@@ -281,10 +292,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             issued_parity[s] = -1;
         bool aborted = false;
         bool first = true;
-        for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-            for (int vt = col; vt < a.n_vt && !aborted; vt += vstep) {
-                const bool two = kTwo && vt + a.G < a.n_vt;
-                const uint32_t stage_tx = 2u * (kStageBytesA + (two ? 2u : 1u) * wb);  // both CTAs' copies
+        for (int mb = grp; mb < a.n_mb && !aborted; mb += mb_step) {
+            const int mb2 = mb + a.n_groups;  // partner row block of a row-pair sweep
+            const bool rows2 = kTwo && mb2 < a.n_mb;
+            for (int vt = col; vt < a.n_vt && !aborted; vt += rows2 ? a.G : vstep) {
+                const bool two = kTwo && (rows2 || vt + a.G < a.n_vt);
+                // both CTAs' copies: H, the tile's W, and the partner block's H or the second tile's W
+                const uint32_t stage_tx = 2u * (kStageBytesA + wb + (rows2 ? kStageBytesA : (two ? wb : 0u)));
                 for (int kb = 0; kb < a.n_kb; ++kb) {
                     int ok = 1;
                     if (lane == 0)
@@ -301,7 +315,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         ptx::tma_load_2d_pair(sA(stage), &tmH, bar, kb * kBK, mb * kPairM + (int)rank * kBM, pol_h);
                         ptx::tma_load_2d_pair(sB(stage, 0), &tmW, bar, w_x(kb),
                                               w_y(kb, vt * a.bn + (int)rank * half_bn), pol_w);
-                        if (two)
+                        if (rows2)
+                            ptx::tma_load_2d_pair(sB(stage, 1), &tmH, bar, kb * kBK,
+                                                  mb2 * kPairM + (int)rank * kBM, pol_h);
+                        else if (two)
                             ptx::tma_load_2d_pair(sB(stage, 1), &tmW, bar, w_x(kb),
                                                   w_y(kb, (vt + a.G) * a.bn + (int)rank * half_bn), pol_w);
                         if (tl && first)
@@ -341,16 +358,25 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 ptx::tc_fence_after();
                 return ok != 0;
             };
-            auto issue = [&](int acc, int s, int tile, int kb) {  // 4 x K16 of one tile from stage s
-                const uint64_t da = ptx::sdesc_kmajor_sw128(sA(s));
-                const uint64_t db = ptx::sdesc_kmajor_sw128(sB(s, tile));
+            auto issue = [&](int acc, uint32_t a_smem, uint32_t b_smem, int kb) {  // 4 x K16 from one stage
+                const uint64_t da = ptx::sdesc_kmajor_sw128(a_smem);
+                const uint64_t db = ptx::sdesc_kmajor_sw128(b_smem);
 #pragma unroll
                 for (int k = 0; k < kBK / 16; ++k)  // +32 B along K per MMA = +2 in the encoded address
                     ptx::mma_bf16_pair(tmem + (uint32_t)acc * kBN, da + 2u * k, db + 2u * k, idesc, (kb | k) != 0);
             };
-            for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-                for (int vt = col; vt < a.n_vt && !aborted; vt += vstep, ++item) {
-                    const bool two = kTwo && vt + a.G < a.n_vt;
+            for (int mb = grp; mb < a.n_mb && !aborted; mb += mb_step) {
+                const bool rows2 = kTwo && mb + a.n_groups < a.n_mb;
+                // accumulator 1 of a pass: the partner block's H (third slot) x the tile's W, or this block's
+                // H x the second tile's W (third slot)
+                auto issue1 = [&](int s, int kb) {
+                    if (rows2)
+                        issue(1, sB(s, 1), sB(s, 0), kb);
+                    else
+                        issue(1, sA(s), sB(s, 1), kb);
+                };
+                for (int vt = col; vt < a.n_vt && !aborted; vt += rows2 ? a.G : vstep, ++item) {
+                    const bool two = kTwo && (rows2 || vt + a.G < a.n_vt);
                     // single tiles: item i uses accumulator i & 1 for the (i >> 1)-th time;
                     // passes: item i uses both accumulators for the i-th time
                     const int acc0 = kTwo ? 0 : (item & 1);
@@ -359,7 +385,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         aborted = true;
                         break;
                     }
-                    const int defer = two ? min(S, a.n_kb) : 0;  // stages whose second-tile MMAs wait
+                    const int defer = two ? min(S, a.n_kb) : 0;  // stages whose second-accumulator MMAs wait
                     const int s0 = stage;
                     for (int kb = 0; kb < a.n_kb; ++kb) {
                         int ok = 1;
@@ -372,7 +398,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         }
                         ptx::tc_fence_after();
                         if (lane == 0)
-                            issue(acc0, stage, 0, kb);
+                            issue(acc0, sA(stage), sB(stage, 0), kb);
                         if (kb < defer) {
                             if (kb == defer - 1) {  // the second accumulator is needed now
                                 if (!wait_acc_free(1, (uint32_t)item)) {
@@ -382,13 +408,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                                 if (lane == 0)
                                     for (int j = 0; j < defer; ++j) {
                                         const int sj = (s0 + j) % S;
-                                        issue(1, sj, 1, j);
+                                        issue1(sj, j);
                                         ptx::mma_commit_pair_multicast(empty(sj), kBothCtas);
                                     }
                             }
                         } else if (lane == 0) {
                             if (two)
-                                issue(1, stage, 1, kb);
+                                issue1(stage, kb);
                             ptx::mma_commit_pair_multicast(empty(stage), kBothCtas);
                         }
                         __syncwarp();
@@ -439,11 +465,17 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             if (lane == 0)
                 ptx::mbar_arrive_cluster(ptx::mapa(tempty(i), 0));
         };
-        for (int mb = grp; mb < a.n_mb && !aborted; mb += a.n_groups) {
-            const int64_t row = (int64_t)mb * kPairM + (int)rank * kBM + q * 32 + lane;
+        const RowState r0{-INFINITY, 0.f, 0.f, 0.f, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0};
+        for (int mb = grp; mb < a.n_mb && !aborted; mb += mb_step) {
+            const int mb2 = mb + a.n_groups;
+            const bool rows2 = kTwo && mb2 < a.n_mb;
+            const int64_t in_block = (int)rank * kBM + q * 32 + lane;
+            const int64_t row = (int64_t)mb * kPairM + in_block;
+            const int64_t row2 = rows2 ? (int64_t)mb2 * kPairM + in_block : (int64_t)a.N;  // a.N: no row
             const int32_t tgt = (row < a.N) ? row_target(a.ts, row, a.V) : -1;
-            RowState r{-INFINITY, 0.f, 0.f, 0.f, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0};
-            for (int vt = col; vt < a.n_vt; vt += vstep, ++item) {
+            const int32_t tgt2 = (row2 < a.N) ? row_target(a.ts, row2, a.V) : -1;
+            RowState r = r0, r2 = r0;  // r2: the partner block's row in a row-pair sweep
+            for (int vt = col; vt < a.n_vt; vt += rows2 ? a.G : vstep, ++item) {
                 const int acc0 = kTwo ? 0 : (item & 1);
                 const uint32_t uses0 = kTwo ? (uint32_t)item : (uint32_t)(item >> 1);
                 if (!take(acc0, uses0)) {
@@ -458,20 +490,27 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                         break;
                     }
                     const int vt1 = vt + a.G;
-                    if (vt1 < a.n_vt)
+                    if (rows2)
+                        fold_tile<kEntropy>(r2, lanes + kBN, vt * a.bn, min(a.bn, a.V - vt * a.bn), tgt2);
+                    else if (vt1 < a.n_vt)
                         fold_tile<kEntropy>(r, lanes + kBN, vt1 * a.bn, min(a.bn, a.V - vt1 * a.bn), tgt);
                     release(1);
                 }
             }
-            if (!aborted && row < a.N) {
-                if (pend_idx >= 0) {
-                    a.part[pend_idx] = pend;
+            if (aborted)
+                break;
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {  // the previous sweep's records, then this sweep's become pending
+                if (pend_idx[i] >= 0) {
+                    a.part[pend_idx[i]] = pend[i];
                     if (kEntropy)
-                        a.part_u[pend_idx] = pend_u;
+                        a.part_u[pend_idx[i]] = pend_u[i];
                 }
-                pend = make_float4(r.m, (r.s0 + r.s1) + (r.s2 + r.s3), __int_as_float(r.am), r.tlog);
-                pend_u = (r.u0 + r.u1) + (r.u2 + r.u3);
-                pend_idx = row * a.G + col;
+                const RowState &x = i ? r2 : r;
+                pend[i] = make_float4(x.m, (x.s0 + x.s1) + (x.s2 + x.s3), __int_as_float(x.am), x.tlog);
+                pend_u[i] = (x.u0 + x.u1) + (x.u2 + x.u3);
+                const int64_t rr = i ? row2 : row;
+                pend_idx[i] = rr < a.N ? rr * a.G + col : -1;
             }
         }
         if (tl && !leader && warp == 2 && lane == 0)
@@ -484,11 +523,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     if (tl && threadIdx.x == 0)
         tl[5] = ptx::globaltimer_ns();
     ptx::cluster_arrive_release();
-    if (pend_idx >= 0) {
-        a.part[pend_idx] = pend;
-        if (kEntropy)
-            a.part_u[pend_idx] = pend_u;
-    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+        if (pend_idx[i] >= 0) {
+            a.part[pend_idx[i]] = pend[i];
+            if (kEntropy)
+                a.part_u[pend_idx[i]] = pend_u[i];
+        }
     if (threadIdx.x == 64) {
         // Warp 2 has passed griddepcontrol.wait, so the previous call's finish kernel, which clears the
         // status word, has completed: a failure recorded now belongs to this call.
@@ -547,7 +588,11 @@ ScoreSchedule score_schedule(int32_t n_mb, int64_t V, int max_units, int32_t rec
             }
         }
     }
-    best.stage_bytes = kStageBytesA + (uint32_t)(1 + two) * stage_bytes_w(best.bn);
+    // A pass stage has a third slot: the second tile's W, or in a row-pair sweep (a group with more than
+    // one row block) the partner block's H.
+    const uint32_t wb = stage_bytes_w(best.bn);
+    const bool row_pairs = two && n_mb > best.n_groups;
+    best.stage_bytes = kStageBytesA + wb + (two ? (row_pairs && wb < kStageBytesA ? kStageBytesA : wb) : 0u);
     const uint32_t fit = kRingCapacity / best.stage_bytes;
     best.stages = (int32_t)(fit < (uint32_t)kMaxStages ? fit : (uint32_t)kMaxStages);
     return best;
@@ -611,6 +656,13 @@ cudaError_t launch_score(const CUtensorMap &tmH, const CUtensorMap &tmW, const S
 {
     if (configure_device() < 1)
         return cudaErrorUnknown;
+    // The ring must hold what the producer stages: a pass's third slot takes an H box (16 KB) in a row-pair
+    // sweep, which the launch has when a group owns more than one row block.
+    const uint32_t wb = stage_bytes_w(a.bn);
+    const uint32_t third = a.two ? (a.n_mb > a.n_groups && wb < kStageBytesA ? kStageBytesA : wb) : 0u;
+    if (a.stages < 2 || a.stages > kMaxStages || a.stage_bytes < kStageBytesA + wb + third ||
+        a.stage_bytes % 1024u != 0 || (uint64_t)a.stages * a.stage_bytes > kRingCapacity)
+        return cudaErrorInvalidValue;
     cudaLaunchAttribute attr[2];
     cudaLaunchConfig_t cfg = score_config((unsigned)(2 * a.n_groups * a.G),
                                           kSmemOverhead + (uint32_t)a.stages * a.stage_bytes, stream, attr);

@@ -48,7 +48,11 @@ def test_split_invariants(sm, pairs):
         assert p["n_groups"] * p["G"] <= units and p["ctas"] == 2 * p["n_groups"] * p["G"], p
         assert p["records_per_row"] == min(math.ceil(V / 128), 256), p
         assert p["two"] == (1 if p["n_mb"] >= 2 else 0), p
-        assert p["stage_bytes"] == 16384 + (1 + p["two"]) * p["bn"] * 64, p
+        wb = p["bn"] * 64  # W bytes per CTA and K slice of one tile
+        # a pass stage's third slot: the second tile's W, or the partner row block's H (16 KB) when a group
+        # owns more than one row block (row-pair sweeps)
+        third = (16384 if p["n_mb"] > p["n_groups"] and wb < 16384 else wb) if p["two"] else 0
+        assert p["stage_bytes"] == 16384 + wb + third, p
         ring = p["stages"] * p["stage_bytes"]
         assert 2 <= p["stages"] <= 7 and ring + SMEM_OVERHEAD <= SMEM_MAX, p
         assert 2 * (ring + SMEM_OVERHEAD) > SM_SHARED, p  # never two CTAs (two TMEM owners) on one SM
@@ -56,13 +60,47 @@ def test_split_invariants(sm, pairs):
         assert wino.wino_workspace_size(N, 4096, V) >= N * p["G"] * 16
 
 
-@pytest.mark.parametrize("N,V", [(64, 1000), (256, 126464), (300, 5000), (1024, 126464), (2048, 134400),
-                                 (4096, 32641), (8192, 1000)])
+def _walk(plan):
+    """The items each CTA pair computes, in the order the score kernel's three roles walk them: per pair a
+    list of items, each a list of (row block, tile, accumulator); and the vocabulary sweeps per group."""
+    pairs = plan["ctas"] // 2
+    ng, G, n_mb, n_vt, two = plan["n_groups"], plan["G"], plan["n_mb"], plan["n_vt"], plan["two"]
+    items, sweeps = {}, {}
+    for c in range(pairs):
+        grp, col = c % ng, c // ng
+        out = items.setdefault(c, [])
+        for mb in range(grp, n_mb, 2 * ng if two else ng):
+            sweeps[grp] = sweeps.get(grp, 0) + (1 if col == 0 else 0)
+            mb2 = mb + ng
+            if two and mb2 < n_mb:  # row-pair sweep: one tile of both blocks per item
+                for vt in range(col, n_vt, G):
+                    out.append([(mb, vt, 0), (mb2, vt, 1)])
+            elif two:  # tile-pair sweep of a block without a partner
+                for vt in range(col, n_vt, 2 * G):
+                    out.append([(mb, vt, 0)] + ([(mb, vt + G, 1)] if vt + G < n_vt else []))
+            else:  # single tiles, alternating accumulators
+                for vt in range(col, n_vt, G):
+                    out.append([(mb, vt, len(out) & 1)])
+    return items, sweeps
+
+
+@pytest.mark.parametrize("N,V", [(64, 1000), (256, 126464), (300, 5000), (768, 126464), (1024, 126464),
+                                 (1280, 126464), (2048, 134400), (4096, 32641), (8192, 1000)])
 def test_every_tile_once_and_balanced(N, V):
     p = wino.wino_score_plan_host(N, 4096, V)
     own = _owners(p)
     assert sorted(own) == sorted(itertools.product(range(p["n_mb"]), range(p["n_vt"])))
     assert all(len(v) == 1 for v in own.values())
+    # the kernel's walk computes the same (row block, tile) set, each once, both accumulators of a pass
+    # holding different tiles
+    items, sweeps = _walk(p)
+    walked = [(mb, vt) for its in items.values() for it in its for mb, vt, _ in it]
+    assert sorted(walked) == sorted(own)
+    assert all(len({acc for _, _, acc in it}) == len(it) for its in items.values() for it in its)
+    # with passes, a group sweeps the vocabulary (reads W) once per two of its row blocks
+    if p["two"]:
+        for g in range(p["n_groups"]):
+            assert sweeps[g] == math.ceil(len(range(g, p["n_mb"], p["n_groups"])) / 2)
     for g in range(p["n_groups"]):  # within a group, tiles per pair and row block differ by at most one
         counts = [len(range(c // p["n_groups"], p["n_vt"], p["G"])) for c in range(g, p["ctas"] // 2, p["n_groups"])]
         assert max(counts) - min(counts) <= 1
@@ -76,6 +114,7 @@ def test_benchmark_shapes():
         b8 = wino.wino_score_plan_host(2048, 4096, V)
         assert (b8["bn"], b8["n_groups"], b8["G"], b8["two"], b8["stages"]) == (256, 4, 19, 1, 4)
         assert math.ceil(b8["n_vt"] / b8["G"]) == tiles
+        assert b8["n_mb"] == 2 * b8["n_groups"]  # one row-pair sweep per group: W is read once
     loop = wino.wino_score_plan_host(1024, 4096, 126464)
     assert (loop["bn"], loop["n_groups"], loop["G"], loop["two"]) == (256, 4, 19, 1)
 
