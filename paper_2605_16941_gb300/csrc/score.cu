@@ -549,13 +549,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 }  // namespace
 
 // Choose the mode, the tile width bn and the number of row-block groups.  One 256-row block is bound by the
-// W stream from HBM: single tiles (the most bytes in flight).  More rows are tensor-bound: two-tile passes
-// (fewer bytes delivered per MMA).  Then: fewest vocabulary columns on the busiest pair plus a per-tile or
+// W stream from HBM: single tiles (the most bytes in flight).  More rows are tensor-bound: passes (fewer bytes
+// delivered per MMA; row-pair sweeps where a group owns more than one row block).  Then: fewest vocabulary columns on the busiest pair plus a per-tile or
 // per-pass overhead, the widest tile, fewest passes over W (more groups).  A width below kBN pays when the
 // vocabulary then splits evenly over the pairs: V = 126464 on 76 pairs is 494 tiles of 256 (7 on the
 // busiest pair, 6.5 on average) but 527 tiles of 240 (7 on 71 pairs).
 #ifndef WINO_PASS_MIN_ROW_BLOCKS
-#define WINO_PASS_MIN_ROW_BLOCKS 2  // compile-time tuning: fewest 256-row blocks that use two-tile passes
+#define WINO_PASS_MIN_ROW_BLOCKS 2  // compile-time tuning: fewest 256-row blocks that use passes
 #endif
 constexpr int32_t kPassMinRowBlocks = WINO_PASS_MIN_ROW_BLOCKS;
 

@@ -3,7 +3,7 @@
 The copy must be the stated permutation of W, bit for bit, and a step that reads W through it must give the same
 bytes as the step over row-major W: the score kernel then multiplies the same operands in the same order, so the
 token state, the counts, the flags and the whole workspace (partial softmax records, per-row statistics, status
-words) are compared for equality, in single-tile launches (one 256-row block), two-tile passes (N = 2048) and
+words) are compared for equality, in single-tile launches (one 256-row block), passes (N = 2048) and
 with ragged vocabulary and row tails.  The row-major step itself is compared with the oracle elsewhere."""
 import dataclasses
 
@@ -52,9 +52,9 @@ def _assert_same(a, b):
         assert torch.equal(x, y), f"{what} differ between row-major W and its panel copy"
 
 
-# tiny (N = 64), a ragged shape (V % 240 and N % 256 both non-zero, three row blocks: two-tile passes with a
+# tiny (N = 64), a ragged shape (V % 240 and N % 256 both non-zero, three row blocks: tile-pair passes with a
 # single-tile remainder), the LLaDA single step (N = 256, bn = 240) and its coverage variant, and the
-# unified-vocabulary step (N = 2048, V = 134400, two-tile passes)
+# unified-vocabulary step (N = 2048, V = 134400, row-pair passes)
 RAGGED = ws.Workload("panels_ragged", d=128, V=5003, n_seq=5, blk_len=56, bias=((1.0, 0.0, 9.0),), predecoded=0.4,
                      hold=0.5, tau1=0.6, tau2=0.8)
 

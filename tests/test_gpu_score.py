@@ -18,11 +18,17 @@ SHAPES = [
     (384, 520, 777),
     (100, 64, 19400),   # last pair: one 256-wide tile with 200 valid columns
     (256, 128, 50000),  # several 256-wide tiles per pair and a 128-wide tail tile
-    # two-tile passes (two or more 256-row blocks):
+    # passes (two or more 256-row blocks), tile-pair sweeps (one row block per group):
     (512, 64, 40000),   # one K slice: the second accumulator's MMAs deferred over a one-stage window
     (520, 8, 300),      # d = 8 (K slice mostly zero fill), ragged last row block
     (2048, 64, 129),    # a vocabulary narrower than one tile: every pass holds a single tile
     (1024, 192, 70000),  # many passes per pair, odd tile counts (a single-tile last pass), ragged vocabulary
+    # row-pair sweeps (groups owning two or more row blocks; the third stage slot holds an H box):
+    (2400, 64, 5000),   # 5 groups x 2 blocks, bn = 176; the ragged last block is a partner whose second
+                        # CTA's rows all lie past N
+    (2000, 64, 20000),  # 4 groups x 2 blocks, ragged partner block with rows in both CTAs
+    (1300, 64, 20000),  # 2 groups x 3 blocks: a row-pair sweep, then the ragged third block alone
+    (3100, 64, 20000),  # 2 groups x 7 / 6 blocks: several row-pair sweeps per pair (records of each sweep)
 ]
 
 
