@@ -369,9 +369,11 @@ WINO_API int wino_timeline_end(int64_t *launches);
  * (diagnostics; the paper has no counterpart): plan (host int32[8]) receives
  * the tile width bn, the vocabulary tiles n_vt = ceil(V / bn), the 256-row
  * blocks n_mb, the row-block groups, the CTA pairs per group G (= records per
- * row), the grid size in CTAs, 1 if tiles are taken two per pass (one staging
- * of H for both) else 0, and the shared-memory ring stages.  Pair c of the
- * launch serves row blocks c % groups (+ groups, ...) and, within each, tiles
+ * row), the grid size in CTAs, 1 if the kernel works in passes (each staged
+ * slice feeds both accumulators: two row blocks of a group share a tile's W
+ * slice, or a row block left without a partner shares its H slice between two
+ * tiles) else 0, and the shared-memory ring stages.  Pair c of the launch
+ * serves row blocks c % groups (+ groups, ...) and, within each, tiles
  * c / groups (+ G, ...).
  */
 WINO_API int wino_score_plan(int64_t N, int64_t d, int64_t V, int32_t *plan);
